@@ -1,0 +1,284 @@
+/*
+ * libispa -- the data-parallel hot path of ISPA (Instance-Specific Parametric
+ * Absorption, arxiv 2607.00712) on one GB300 (sm_103a).
+ *
+ * The library computes, for one transformer layer of an autoregressive video
+ * DiT and one chunk step:
+ *   - F-layer attention over the whole KV cache (Sec. 2, Eq. 3);
+ *   - L-layer attention over a sink + recent-frame window (Sec. 3.3, Eq. 7);
+ *   - the dual warmup pass returning both outputs from one sweep over the key
+ *     tiles, with their per-token discrepancy (Sec. 3.1, Sec. 3.4, Eq. 9-12);
+ *   - the running sums of the least-squares absorption (Sec. 3.2, Eq. 5) and
+ *     the closed-form solve with its feasibility score (Eq. 5-6);
+ *   - appending a finished chunk's K/V into a ring-buffer cache.
+ *
+ * Conventions (all entry points)
+ *   - Every tensor argument is a DEVICE pointer owned by the caller, unless
+ *     the argument says "host".  The library allocates no device memory;
+ *     calls that need scratch take a caller workspace and have a size query.
+ *   - bf16 = IEEE bfloat16 stored as 16-bit words.  Layouts are row-major,
+ *     dense, innermost index last.  Device pointers must be 16-byte aligned.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is the
+ *     legacy default stream) except where a function says it synchronises.
+ *   - Errors are returned as ispa_status; no exception crosses the ABI.  On a
+ *     non-OK return of argument validation nothing has been enqueued.
+ *   - Kernels never spin without bound: a wait that runs out records a device
+ *     error, which ispa_last_device_error() reports as ISPA_ERR_TIMEOUT.
+ *   - Head dims supported: 64 and 128.  Tokens per frame P >= 1.
+ */
+#ifndef ISPA_H_
+#define ISPA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ISPA_API __attribute__((visibility("default")))
+#else
+#define ISPA_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ispa_stream; /* == cudaStream_t */
+
+typedef enum {
+  ISPA_OK = 0,
+  ISPA_ERR_INVALID_ARG = 1, /* null/misaligned pointer, bad size or layout */
+  ISPA_ERR_UNSUPPORTED = 2, /* head_dim or hidden size the kernels do not handle */
+  ISPA_ERR_CAPACITY = 3,    /* window or append does not fit the ring */
+  ISPA_ERR_NOT_SPD = 4,     /* Gram matrix + lambda I not positive definite */
+  ISPA_ERR_TIMEOUT = 5,     /* a device-side bounded wait ran out */
+  ISPA_ERR_CUDA = 6,        /* a CUDA runtime/driver call failed */
+  ISPA_ERR_WORKSPACE = 7    /* workspace missing or smaller than the size query */
+} ispa_status;
+
+/*
+ * Per-layer KV cache as a frame-granular ring (Sec. 2: "truncated to include
+ * only the KV pairs from the most recent frames"; Sec. 3.4: sink frame K_1).
+ *   k, v : bf16 [num_heads][capacity_frames * tokens_per_frame][head_dim],
+ *          caller-owned device memory of ispa_ring_bytes()/2 bytes each.
+ *   Logical frame f (0, 1, 2, ... in generation order) lives in slot
+ *     f                                              if f <  n_sink_frames,
+ *     n_sink_frames + (f - n_sink_frames) mod (capacity_frames - n_sink_frames)
+ *                                                    otherwise,
+ *   so the first n_sink_frames frames are pinned and every later frame
+ *   overwrites the oldest non-sink frame.  frames_written counts the frames
+ *   appended so far; it is advanced on the host by ispa_kv_append when the
+ *   copy is enqueued.  The struct is plain data: copying it (and the two
+ *   buffers) checkpoints the cache.
+ */
+typedef struct {
+  int32_t num_heads;
+  int32_t head_dim;
+  int32_t tokens_per_frame;
+  int32_t capacity_frames;
+  int32_t n_sink_frames;
+  int32_t reserved;
+  int64_t frames_written;
+  void* k;
+  void* v;
+} ispa_kv_ring;
+
+/*
+ * Local window of an L-layer (Eq. 7, read as a parameterised window): the
+ * n_sink_frames oldest past frames plus the n_recent_frames newest past
+ * frames; the chunk itself is always local.  The paper-literal set is
+ * {n_sink_frames = 1, n_recent_frames = 0}.
+ */
+typedef struct {
+  int32_t n_sink_frames;
+  int32_t n_recent_frames;
+} ispa_window;
+
+typedef struct {
+  int32_t first_slot;
+  int32_t n_slots;
+} ispa_slot_range;
+
+#define ISPA_MAX_RANGES 4
+
+/* Slot runs of the full, local and history key sets of a ring (Eq. 7-8). */
+typedef struct {
+  int32_t n_full, n_local, n_hist, reserved;
+  ispa_slot_range full[ISPA_MAX_RANGES];
+  ispa_slot_range local[ISPA_MAX_RANGES];
+  ispa_slot_range hist[ISPA_MAX_RANGES];
+} ispa_key_sets;
+
+/*
+ * Least-squares accumulators (Sec. 3.2: "summing the outer products of
+ * activations").  gram: caller-owned fp32 [2*dim][2*dim], row-major, holding
+ * the blocks of [A_loc | Delta]^T [A_loc | Delta] with Delta = A_full - A_loc:
+ *   G = A_loc^T A_loc   rows [0,dim)     cols [0,dim)
+ *   X = A_loc^T Delta   rows [0,dim)     cols [dim,2dim)
+ *   S = Delta^T Delta   rows [dim,2dim)  cols [dim,2dim)
+ * Only the upper 128x128 tiles of G and S (diagonal tiles in full) and all of
+ * X are maintained; the rest of the buffer is left untouched.  The paper's
+ * A_loc^T R equals X W and is formed by the solve.  n_tokens counts the rows
+ * accumulated (host side).  Plain data: copying it checkpoints the warmup.
+ */
+typedef struct {
+  int32_t dim;
+  int32_t reserved;
+  int64_t n_tokens;
+  float* gram;
+} ispa_ls_state;
+
+/* ------------------------------------------------------------ misc / host */
+
+/* Static English name of a status code. */
+ISPA_API const char* ispa_status_string(ispa_status s);
+
+/* Device error recorded by a kernel on the current device since the last
+ * call (then cleared): ISPA_OK or ISPA_ERR_TIMEOUT.  Synchronises the device
+ * with a blocking copy of one word.  *code (nullable, host) gets the raw code. */
+ISPA_API ispa_status ispa_last_device_error(int32_t* code);
+
+/* Bound of every device-side wait, in nanoseconds (default 1e9).  Applies to
+ * launches enqueued after the call.  Returns the previous value.  Meant for
+ * tests of the timeout path; 0 restores the default. */
+ISPA_API uint64_t ispa_set_wait_limit_ns(uint64_t ns);
+
+/* Enqueue one CTA that waits on an mbarrier nobody arrives at, with the given
+ * bound; it records ISPA_ERR_TIMEOUT and exits.  Exercises the bounded-wait
+ * and status path without touching any other state. */
+ISPA_API ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream);
+
+/* Bytes of one ring's K and V buffers together (2 * H * cap * P * d * 2). */
+ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);
+
+/* Host-only: ring slot of logical frame `frame` (see ispa_kv_ring), or -1 if
+ * the frame is not resident. */
+ISPA_API int32_t ispa_ring_slot(const ispa_kv_ring* ring, int64_t frame);
+
+/*
+ * Host-only (Eq. 7-8): resolve the key sets of the ring's current state.
+ * With F = frames_written, local past frames are {f < win.n_sink_frames}
+ * united with {F - win.n_recent_frames <= f < F}; full = every resident
+ * frame; hist = full minus local.  Each set is returned as increasing runs of
+ * ring slots.  Errors: ISPA_ERR_CAPACITY if a local frame has been evicted,
+ * ISPA_ERR_INVALID_ARG on a bad ring or window.
+ */
+ISPA_API ispa_status ispa_window_resolve(const ispa_kv_ring* ring, ispa_window win, ispa_key_sets* out);
+
+/* ------------------------------------------------------------ KV append */
+
+/*
+ * Write a finished chunk's keys and values into the ring (Eq. 3's K_past
+ * grows by the chunk) and advance ring->frames_written by n_frames.
+ *   k_new, v_new : bf16 [n_frames * P][num_heads][head_dim] (token-major, as
+ *                  produced by the QKV projection).
+ * Frame frames_written + i goes to its ring slot, evicting the oldest non-sink
+ * frame.  Errors: ISPA_ERR_CAPACITY if n_frames > capacity - n_sink (a frame
+ * of this append would overwrite another one of it) or n_frames > 16.
+ */
+ISPA_API ispa_status ispa_kv_append(ispa_kv_ring* ring, const void* k_new, const void* v_new,
+                           int32_t n_frames, ispa_stream stream);
+
+/* Same for n_layers rings in ONE launch.  The rings share num_heads,
+ * head_dim and tokens_per_frame; capacity, sinks and frames_written may differ.
+ * rings: host array of n_layers ring structs (each advanced); k_new/v_new:
+ * host arrays of n_layers device pointers.  n_layers <= 64. */
+ISPA_API ispa_status ispa_kv_append_layers(ispa_kv_ring* rings, int32_t n_layers,
+                                  const void* const* k_new, const void* const* v_new,
+                                  int32_t n_frames, ispa_stream stream);
+
+/* ------------------------------------------------------------ attention */
+
+/*
+ * F-layer chunk attention (Eq. 3): Q = Q_cur, K = [K_past; K_cur],
+ * V = [V_past; V_cur], with K_past/V_past every resident frame of the ring.
+ * The chunk is dense inside itself (no intra-chunk mask).
+ *   q, k_cur, v_cur : bf16 [n_q][num_heads][head_dim]
+ *   out             : bf16 [n_q][num_heads * head_dim]  (heads concatenated)
+ *   lse             : fp32 [num_heads][n_q], natural-log LSE, or NULL
+ *   scale           : softmax scale; 0 means 1/sqrt(head_dim)
+ * Computation: bf16 inputs, fp32 accumulation, bf16 output (round to nearest).
+ */
+ISPA_API ispa_status ispa_attn_full(const ispa_kv_ring* ring, const void* q, const void* k_cur,
+                           const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
+                           ispa_stream stream);
+
+/*
+ * L-layer chunk attention (Sec. 3.3, Eq. 7): the same over the local set
+ * only -- the window's sink and recent frames plus the chunk.  Arguments as
+ * for ispa_attn_full.  Errors: ISPA_ERR_CAPACITY if a window frame has been
+ * evicted from the ring.
+ */
+ISPA_API ispa_status ispa_attn_local(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                            const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                            void* out, float* lse, ispa_stream stream);
+
+/* Workspace bytes of ispa_attn_dual (fp32 [num_heads][n_q] partial sums). */
+ISPA_API size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q);
+
+/*
+ * Warmup dual pass (Sec. 3.1 phase 1, Sec. 3.4): A_loc (local set) and A_full
+ * (full set) of the same queries from one sweep over the key tiles -- the
+ * local tiles first, then the history tiles, fusing the two online-softmax
+ * states as Eq. 11-12 do.
+ *   a_full, a_loc  : bf16 [n_q][num_heads * head_dim]
+ *   disc           : fp32 [n_q], disc_t = || A_full,t - A_loc,t ||_2 over all
+ *                    num_heads*head_dim features, taken on the stored bf16
+ *                    outputs (the paper's "output discrepancy", read as this norm)
+ *   disc_sq_sum    : fp32 device scalar, += sum_t disc_t^2 (not reset)
+ *   lse_full, lse_loc : fp32 [num_heads][n_q] or NULL
+ *   workspace      : >= ispa_attn_dual_workspace_size bytes
+ * An empty history set gives a_full == a_loc bit for bit and disc == 0.
+ */
+ISPA_API ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                           const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                           void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                           float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                           ispa_stream stream);
+
+/* ------------------------------------------------------------ least squares */
+
+/* Bytes of the fp32 [2*dim][2*dim] gram buffer. */
+ISPA_API size_t ispa_ls_state_bytes(int32_t dim);
+
+/* Zero state->gram (async) and state->n_tokens. */
+ISPA_API ispa_status ispa_ls_state_reset(ispa_ls_state* state, ispa_stream stream);
+
+/* Workspace bytes of ispa_ls_accumulate for T tokens of width dim. */
+ISPA_API size_t ispa_ls_accumulate_workspace_size(int32_t dim, int64_t T);
+
+/*
+ * Add T tokens to the normal-equation sums (Sec. 3.2, "summing the outer
+ * products ... during the standard forward pass"):
+ *   G += A_loc^T A_loc,  X += A_loc^T Delta,  S += Delta^T Delta,  n += T,
+ * Delta = A_full - A_loc taken exactly in fp32 and carried as a bf16 hi + lo
+ * pair, products on the tensor cores with fp32 accumulation.
+ *   a_loc, a_full : bf16 [T][dim], dim a multiple of 128 (else UNSUPPORTED).
+ */
+ISPA_API ispa_status ispa_ls_accumulate(ispa_ls_state* state, const void* a_loc, const void* a_full,
+                               int64_t T, void* workspace, size_t ws_bytes, ispa_stream stream);
+
+/* Workspace bytes of ispa_ls_solve. */
+ISPA_API size_t ispa_ls_solve_workspace_size(int32_t dim, int32_t d_out);
+
+/*
+ * Closed-form absorption (Eq. 5) and feasibility score (Eq. 6), fp64:
+ *   dW  = (G + lambda I)^{-1} X W          (Cholesky solve, Eq. 5 with R = Delta W)
+ *   eps = || A_loc (W + dW) - A_full W ||_F^2
+ *       = tr(W^T S W) - ||L^{-1} X W||_F^2 - lambda ||dW||_F^2,  L L^T = G + lambda I.
+ *   W       : fp32 [dim][d_out], row-vector convention (out = A @ W; a torch
+ *             nn.Linear weight is W^T)
+ *   dW      : fp32 [dim][d_out] output
+ *   eps_out : HOST double (nullable)
+ *   lambda  : ridge weight on the unnormalised sums (paper default 1e-3)
+ * Synchronises `stream`.  Errors: ISPA_ERR_NOT_SPD if a Cholesky pivot is not
+ * positive.
+ */
+ISPA_API ispa_status ispa_ls_solve(const ispa_ls_state* state, const float* W, int32_t d_out,
+                          double lambda, float* dW, double* eps_out, void* workspace,
+                          size_t ws_bytes, ispa_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ISPA_H_ */

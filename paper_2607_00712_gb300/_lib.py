@@ -1,0 +1,229 @@
+"""ctypes binding of libispa (include/ispa.h).  Argument marshalling only.
+
+Every function here has the name of the C entry point it calls and passes its
+arguments straight through: tensors become device pointers (``data_ptr()``),
+streams become ``cudaStream_t`` handles, and a non-OK status raises
+``IspaError``.  No computation happens in Python.  If libispa.so is missing
+the import of the library fails loudly; there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, Structure, c_char_p, c_double, c_float, c_int32, c_int64, c_size_t, c_uint64, c_void_p
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libispa.so")
+
+ISPA_OK = 0
+ISPA_ERR_INVALID_ARG = 1
+ISPA_ERR_UNSUPPORTED = 2
+ISPA_ERR_CAPACITY = 3
+ISPA_ERR_NOT_SPD = 4
+ISPA_ERR_TIMEOUT = 5
+ISPA_ERR_CUDA = 6
+ISPA_ERR_WORKSPACE = 7
+MAX_RANGES = 4
+
+
+class KVRing(Structure):
+    _fields_ = [("num_heads", c_int32), ("head_dim", c_int32), ("tokens_per_frame", c_int32),
+                ("capacity_frames", c_int32), ("n_sink_frames", c_int32), ("reserved", c_int32),
+                ("frames_written", c_int64), ("k", c_void_p), ("v", c_void_p)]
+
+
+class Window(Structure):
+    _fields_ = [("n_sink_frames", c_int32), ("n_recent_frames", c_int32)]
+
+
+class SlotRange(Structure):
+    _fields_ = [("first_slot", c_int32), ("n_slots", c_int32)]
+
+
+class KeySets(Structure):
+    _fields_ = [("n_full", c_int32), ("n_local", c_int32), ("n_hist", c_int32), ("reserved", c_int32),
+                ("full", SlotRange * MAX_RANGES), ("local", SlotRange * MAX_RANGES),
+                ("hist", SlotRange * MAX_RANGES)]
+
+    def ranges(self, which: str) -> list[tuple[int, int]]:
+        n = getattr(self, "n_" + which)
+        arr = getattr(self, which)
+        return [(arr[i].first_slot, arr[i].n_slots) for i in range(n)]
+
+
+class LSState(Structure):
+    _fields_ = [("dim", c_int32), ("reserved", c_int32), ("n_tokens", c_int64), ("gram", c_void_p)]
+
+
+class IspaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+_lib = None
+
+# name -> (restype, argtypes)
+_SIGS = {
+    "ispa_status_string": (c_char_p, [c_int32]),
+    "ispa_last_device_error": (c_int32, [POINTER(c_int32)]),
+    "ispa_set_wait_limit_ns": (c_uint64, [c_uint64]),
+    "ispa_debug_wait_probe": (c_int32, [c_uint64, c_void_p]),
+    "ispa_ring_bytes": (c_size_t, [POINTER(KVRing)]),
+    "ispa_ring_slot": (c_int32, [POINTER(KVRing), c_int64]),
+    "ispa_window_resolve": (c_int32, [POINTER(KVRing), Window, POINTER(KeySets)]),
+    "ispa_kv_append": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_int32, c_void_p]),
+    "ispa_kv_append_layers": (c_int32, [POINTER(KVRing), c_int32, POINTER(c_void_p), POINTER(c_void_p),
+                                        c_int32, c_void_p]),
+    "ispa_attn_full": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_int32, c_float, c_void_p,
+                                 c_void_p, c_void_p]),
+    "ispa_attn_local": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
+                                  c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_dual_workspace_size": (c_size_t, [c_int32, c_int32]),
+    "ispa_attn_dual": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
+                                 c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                 c_size_t, c_void_p]),
+    "ispa_ls_state_bytes": (c_size_t, [c_int32]),
+    "ispa_ls_state_reset": (c_int32, [POINTER(LSState), c_void_p]),
+    "ispa_ls_accumulate_workspace_size": (c_size_t, [c_int32, c_int64]),
+    "ispa_ls_accumulate": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
+                                     c_void_p]),
+    "ispa_ls_solve_workspace_size": (c_size_t, [c_int32, c_int32]),
+    "ispa_ls_solve": (c_int32, [POINTER(LSState), c_void_p, c_int32, c_double, c_void_p, POINTER(c_double),
+                                c_void_p, c_size_t, c_void_p]),
+}
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libispa.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libispa.so not built ({LIB_PATH}); run "
+                               "python -m paper_2607_00712_gb300.build")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _ptr(x) -> int | None:
+    """Device pointer of a tensor (or an int / None passed through)."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(s) -> int | None:
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(st: int, where: str) -> None:
+    if st != ISPA_OK:
+        raise IspaError(st, where)
+
+
+def status_string(st: int) -> str:
+    return lib().ispa_status_string(st).decode()
+
+
+def ispa_last_device_error() -> tuple[int, int]:
+    code = c_int32(0)
+    st = lib().ispa_last_device_error(ctypes.byref(code))
+    return st, code.value
+
+
+def ispa_set_wait_limit_ns(ns: int) -> int:
+    return lib().ispa_set_wait_limit_ns(ns)
+
+
+def ispa_debug_wait_probe(limit_ns: int, stream=None) -> None:
+    _check(lib().ispa_debug_wait_probe(limit_ns, _stream(stream)), "ispa_debug_wait_probe")
+
+
+def ispa_ring_bytes(ring: KVRing) -> int:
+    return lib().ispa_ring_bytes(ctypes.byref(ring))
+
+
+def ispa_ring_slot(ring: KVRing, frame: int) -> int:
+    return lib().ispa_ring_slot(ctypes.byref(ring), frame)
+
+
+def ispa_window_resolve(ring: KVRing, win: Window) -> KeySets:
+    ks = KeySets()
+    _check(lib().ispa_window_resolve(ctypes.byref(ring), win, ctypes.byref(ks)), "ispa_window_resolve")
+    return ks
+
+
+def ispa_kv_append(ring: KVRing, k_new, v_new, n_frames: int, stream=None) -> None:
+    _check(lib().ispa_kv_append(ctypes.byref(ring), _ptr(k_new), _ptr(v_new), n_frames, _stream(stream)),
+           "ispa_kv_append")
+
+
+def ispa_kv_append_layers(rings, k_new: list, v_new: list, n_frames: int, stream=None) -> None:
+    """rings: a ctypes array of KVRing (advanced in place)."""
+    n = len(rings)
+    ks = (c_void_p * n)(*[_ptr(x) for x in k_new])
+    vs = (c_void_p * n)(*[_ptr(x) for x in v_new])
+    _check(lib().ispa_kv_append_layers(rings, n, ks, vs, n_frames, _stream(stream)), "ispa_kv_append_layers")
+
+
+def ispa_attn_full(ring: KVRing, q, k_cur, v_cur, n_q: int, scale: float, out, lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_full(ctypes.byref(ring), _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale, _ptr(out),
+                                _ptr(lse), _stream(stream)), "ispa_attn_full")
+
+
+def ispa_attn_local(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, out, lse=None,
+                    stream=None) -> None:
+    _check(lib().ispa_attn_local(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
+                                 _ptr(out), _ptr(lse), _stream(stream)), "ispa_attn_local")
+
+
+def ispa_attn_dual_workspace_size(num_heads: int, n_q: int) -> int:
+    return lib().ispa_attn_dual_workspace_size(num_heads, n_q)
+
+
+def ispa_attn_dual(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, a_full, a_loc, disc,
+                   disc_sq_sum, lse_full=None, lse_loc=None, workspace=None, ws_bytes: int = 0,
+                   stream=None) -> None:
+    _check(lib().ispa_attn_dual(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
+                                _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full),
+                                _ptr(lse_loc), _ptr(workspace), ws_bytes, _stream(stream)), "ispa_attn_dual")
+
+
+def ispa_ls_state_bytes(dim: int) -> int:
+    return lib().ispa_ls_state_bytes(dim)
+
+
+def ispa_ls_state_reset(state: LSState, stream=None) -> None:
+    _check(lib().ispa_ls_state_reset(ctypes.byref(state), _stream(stream)), "ispa_ls_state_reset")
+
+
+def ispa_ls_accumulate_workspace_size(dim: int, T: int) -> int:
+    return lib().ispa_ls_accumulate_workspace_size(dim, T)
+
+
+def ispa_ls_accumulate(state: LSState, a_loc, a_full, T: int, workspace, ws_bytes: int, stream=None) -> None:
+    _check(lib().ispa_ls_accumulate(ctypes.byref(state), _ptr(a_loc), _ptr(a_full), T, _ptr(workspace),
+                                    ws_bytes, _stream(stream)), "ispa_ls_accumulate")
+
+
+def ispa_ls_solve_workspace_size(dim: int, d_out: int) -> int:
+    return lib().ispa_ls_solve_workspace_size(dim, d_out)
+
+
+def ispa_ls_solve(state: LSState, W, d_out: int, lam: float, dW, workspace, ws_bytes: int,
+                  stream=None) -> float:
+    eps = c_double(0.0)
+    _check(lib().ispa_ls_solve(ctypes.byref(state), _ptr(W), d_out, lam, _ptr(dW), ctypes.byref(eps),
+                               _ptr(workspace), ws_bytes, _stream(stream)), "ispa_ls_solve")
+    return eps.value

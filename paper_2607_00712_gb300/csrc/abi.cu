@@ -1,0 +1,452 @@
+// C-ABI entry points of libispa: argument validation, ring bookkeeping
+// (Eq. 7-8 key sets as slot runs), tensor-map encoding and kernel launches.
+// See include/ispa.h for the contract of each function.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+#include <vector>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ispa {
+
+static __device__ int g_status;  // device error word (DEVERR_*), one per device
+
+namespace {
+
+constexpr uint64_t kDefaultWaitLimitNs = 1000ull * 1000 * 1000;
+uint64_t g_wait_limit = kDefaultWaitLimitNs;
+
+bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+}  // namespace
+
+uint64_t wait_limit_ns() { return g_wait_limit; }
+
+int* device_status_ptr() {
+  static int* ptrs[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!ptrs[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+    ptrs[dev] = static_cast<int*>(p);
+  }
+  return ptrs[dev];
+}
+
+bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                    uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
+                    uint32_t b2) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
+                    uint64_t stride1_bytes, uint32_t b0, uint32_t b1) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {d0, d1};
+  cuuint64_t strides[1] = {stride1_bytes};
+  cuuint32_t box[2] = {b0, b1};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ------------------------------------------------------------ ring bookkeeping
+namespace {
+
+ispa_status check_ring(const ispa_kv_ring* r) {
+  if (!r) return ISPA_ERR_INVALID_ARG;
+  if (r->num_heads <= 0 || r->tokens_per_frame <= 0 || r->capacity_frames <= 0 ||
+      r->n_sink_frames < 0 || r->n_sink_frames >= r->capacity_frames || r->frames_written < 0)
+    return ISPA_ERR_INVALID_ARG;
+  if (r->head_dim != 64 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(r->capacity_frames) * r->tokens_per_frame > INT32_MAX)
+    return ISPA_ERR_INVALID_ARG;
+  return ISPA_OK;
+}
+
+bool resident(const ispa_kv_ring* r, int64_t f) {
+  if (f < 0 || f >= r->frames_written) return false;
+  if (f < r->n_sink_frames) return true;
+  return r->frames_written - f <= r->capacity_frames - r->n_sink_frames;
+}
+
+int32_t slot_of(const ispa_kv_ring* r, int64_t f) {
+  if (f < r->n_sink_frames) return static_cast<int32_t>(f);
+  return r->n_sink_frames +
+         static_cast<int32_t>((f - r->n_sink_frames) % (r->capacity_frames - r->n_sink_frames));
+}
+
+// Maximal runs of set entries of a slot mask.
+bool mask_runs(const std::vector<uint8_t>& m, ispa_slot_range* out, int32_t* n) {
+  *n = 0;
+  const int cap = static_cast<int>(m.size());
+  for (int s = 0; s < cap;) {
+    if (!m[s]) {
+      ++s;
+      continue;
+    }
+    int e = s;
+    while (e < cap && m[e]) ++e;
+    if (*n >= ISPA_MAX_RANGES) return false;
+    out[*n].first_slot = s;
+    out[*n].n_slots = e - s;
+    ++*n;
+    s = e;
+  }
+  return true;
+}
+
+ispa_status resolve(const ispa_kv_ring* r, ispa_window win, ispa_key_sets* ks) {
+  if (win.n_sink_frames < 0 || win.n_recent_frames < 0) return ISPA_ERR_INVALID_ARG;
+  memset(ks, 0, sizeof(*ks));
+  const int64_t F = r->frames_written;
+  const int cap = r->capacity_frames;
+  std::vector<uint8_t> full(cap, 0), loc(cap, 0), hist(cap, 0);
+  for (int64_t f = 0; f < std::min<int64_t>(r->n_sink_frames, F); ++f) full[slot_of(r, f)] = 1;
+  for (int64_t f = std::max<int64_t>(r->n_sink_frames, F - (cap - r->n_sink_frames)); f < F; ++f)
+    full[slot_of(r, f)] = 1;
+  auto mark_local = [&](int64_t f) -> bool {
+    if (!resident(r, f)) return false;
+    loc[slot_of(r, f)] = 1;
+    return true;
+  };
+  for (int64_t f = 0; f < std::min<int64_t>(win.n_sink_frames, F); ++f)
+    if (!mark_local(f)) return ISPA_ERR_CAPACITY;
+  for (int64_t f = std::max<int64_t>(0, F - win.n_recent_frames); f < F; ++f)
+    if (!mark_local(f)) return ISPA_ERR_CAPACITY;
+  for (int s = 0; s < cap; ++s) hist[s] = full[s] && !loc[s];
+  if (!mask_runs(full, ks->full, &ks->n_full) || !mask_runs(loc, ks->local, &ks->n_local) ||
+      !mask_runs(hist, ks->hist, &ks->n_hist))
+    return ISPA_ERR_INVALID_ARG;
+  return ISPA_OK;
+}
+
+// ------------------------------------------------------------ attention driver
+enum Mode { MODE_FULL, MODE_LOCAL, MODE_DUAL };
+
+int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
+  int tiles = 0;
+  for (int i = 0; i < n; ++i) {
+    AttnSeg& s = p.seg[p.n_seg++];
+    s.src = src;
+    s.start = r[i].first_slot * P;
+    s.count = r[i].n_slots * P;
+    s.pad = 0;
+    tiles += (s.count + 127) / 128;
+  }
+  return tiles;
+}
+
+ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, const void* q,
+                        const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                        void* out, void* out_loc, float* lse, float* lse_loc, float* disc_part,
+                        cudaStream_t stream) {
+  ispa_status st = check_ring(ring);
+  if (st != ISPA_OK) return st;
+  if (n_q <= 0 || !aligned16(q) || !aligned16(k_cur) || !aligned16(v_cur) || !aligned16(out) ||
+      !aligned16(ring->k) || !aligned16(ring->v))
+    return ISPA_ERR_INVALID_ARG;
+  if (mode == MODE_DUAL && (!aligned16(out_loc) || !disc_part)) return ISPA_ERR_INVALID_ARG;
+  if (!(scale >= 0.f) || !isfinite(scale)) return ISPA_ERR_INVALID_ARG;
+  ispa_key_sets ks;
+  st = resolve(ring, mode == MODE_FULL ? ispa_window{0, 0} : win, &ks);
+  if (st != ISPA_OK) return st;
+
+  const int H = ring->num_heads, HD = ring->head_dim, P = ring->tokens_per_frame;
+  AttnParams p;
+  memset(&p, 0, sizeof(p));
+  p.n_q = n_q;
+  p.num_heads = H;
+  const ispa_slot_range chunk{0, 0};
+  (void)chunk;
+  int tiles = 0;
+  if (mode == MODE_FULL) {
+    tiles += add_segs(p, 0, ks.full, ks.n_full, P);
+  } else {
+    tiles += add_segs(p, 0, ks.local, ks.n_local, P);
+  }
+  {
+    AttnSeg& s = p.seg[p.n_seg++];
+    s.src = 1;
+    s.start = 0;
+    s.count = n_q;
+    tiles += (n_q + 127) / 128;
+  }
+  p.n_local_tiles = tiles;
+  if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P);
+  p.n_tiles = tiles;
+  p.dual = mode == MODE_DUAL ? 1 : 0;
+  const float sc = scale == 0.f ? 1.f / sqrtf(static_cast<float>(HD)) : scale;
+  p.scale_log2 = sc * 1.4426950408889634f;
+  p.wait_limit_ns = g_wait_limit;
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.out_loc = static_cast<__nv_bfloat16*>(out_loc);
+  p.lse = lse;
+  p.lse_loc = lse_loc;
+  p.disc_part = disc_part;
+  p.status = device_status_ptr();
+  if (!p.status) return ISPA_ERR_CUDA;
+
+  const uint64_t row_b = static_cast<uint64_t>(HD) * 2;
+  const uint64_t ring_tok = static_cast<uint64_t>(ring->capacity_frames) * P;
+  CUtensorMap tq, tkr, tvr, tkc, tvc;
+  bool ok = encode_tmap_3d(&tq, q, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
+            encode_tmap_3d(&tkc, k_cur, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
+            encode_tmap_3d(&tvc, v_cur, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
+            encode_tmap_3d(&tkr, ring->k, HD, ring_tok, H, row_b, row_b * ring_tok, 64, 128, 1) &&
+            encode_tmap_3d(&tvr, ring->v, HD, ring_tok, H, row_b, row_b * ring_tok, 64, 128, 1);
+  if (!ok) return ISPA_ERR_CUDA;
+  if (launch_attention(HD, &tq, &tkr, &tvr, &tkc, &tvc, p, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+__global__ void wait_probe_kernel(uint64_t limit_ns, int* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    WaitCtx w{&abort_flag, status, limit_ns};
+    mbar_wait(smem_u32(&bar), 0, w);  // nothing ever arrives: runs out after limit_ns
+  }
+}
+
+}  // namespace
+}  // namespace ispa
+
+using namespace ispa;
+
+extern "C" {
+
+const char* ispa_status_string(ispa_status s) {
+  switch (s) {
+    case ISPA_OK: return "ok";
+    case ISPA_ERR_INVALID_ARG: return "invalid argument";
+    case ISPA_ERR_UNSUPPORTED: return "unsupported shape";
+    case ISPA_ERR_CAPACITY: return "ring capacity exceeded";
+    case ISPA_ERR_NOT_SPD: return "matrix not positive definite";
+    case ISPA_ERR_TIMEOUT: return "device wait timed out";
+    case ISPA_ERR_CUDA: return "CUDA error";
+    case ISPA_ERR_WORKSPACE: return "workspace too small";
+  }
+  return "unknown status";
+}
+
+ispa_status ispa_last_device_error(int32_t* code) {
+  int v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_status, sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
+  const int zero = 0;
+  if (cudaMemcpyToSymbol(g_status, &zero, sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
+  if (code) *code = v;
+  if (v == DEVERR_TIMEOUT) return ISPA_ERR_TIMEOUT;
+  return ISPA_OK;
+}
+
+uint64_t ispa_set_wait_limit_ns(uint64_t ns) {
+  const uint64_t old = g_wait_limit;
+  g_wait_limit = ns == 0 ? kDefaultWaitLimitNs : ns;
+  return old;
+}
+
+ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream) {
+  int* st = device_status_ptr();
+  if (!st) return ISPA_ERR_CUDA;
+  wait_probe_kernel<<<1, 32, 0, stream>>>(limit_ns, st);
+  return cudaGetLastError() == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
+}
+
+size_t ispa_ring_bytes(const ispa_kv_ring* r) {
+  if (!r || r->num_heads <= 0 || r->head_dim <= 0 || r->tokens_per_frame <= 0 || r->capacity_frames <= 0)
+    return 0;
+  return 2ull * r->num_heads * r->capacity_frames * r->tokens_per_frame * r->head_dim * 2ull;
+}
+
+int32_t ispa_ring_slot(const ispa_kv_ring* r, int64_t frame) {
+  if (check_ring(r) == ISPA_ERR_INVALID_ARG || !resident(r, frame)) return -1;
+  return slot_of(r, frame);
+}
+
+ispa_status ispa_window_resolve(const ispa_kv_ring* r, ispa_window win, ispa_key_sets* out) {
+  if (!out) return ISPA_ERR_INVALID_ARG;
+  const ispa_status st = check_ring(r);
+  if (st != ISPA_OK) return st;
+  return resolve(r, win, out);
+}
+
+ispa_status ispa_kv_append_layers(ispa_kv_ring* rings, int32_t n_layers, const void* const* k_new,
+                                  const void* const* v_new, int32_t n_frames, ispa_stream stream) {
+  if (!rings || !k_new || !v_new || n_layers <= 0 || n_layers > kMaxAppendLayers)
+    return ISPA_ERR_INVALID_ARG;
+  if (n_frames <= 0) return ISPA_ERR_INVALID_ARG;
+  const ispa_kv_ring& r0 = rings[0];
+  for (int l = 0; l < n_layers; ++l) {
+    const ispa_status st = check_ring(&rings[l]);
+    if (st != ISPA_OK) return st;
+    const ispa_kv_ring& r = rings[l];
+    if (r.num_heads != r0.num_heads || r.head_dim != r0.head_dim || r.tokens_per_frame != r0.tokens_per_frame)
+      return ISPA_ERR_INVALID_ARG;
+    if (!aligned16(r.k) || !aligned16(r.v) || !aligned16(k_new[l]) || !aligned16(v_new[l]))
+      return ISPA_ERR_INVALID_ARG;
+    if (n_frames > kMaxAppendFrames || n_frames > r.capacity_frames - r.n_sink_frames) return ISPA_ERR_CAPACITY;
+  }
+  if (static_cast<int64_t>(n_frames) * r0.tokens_per_frame * r0.num_heads * (r0.head_dim / 8) >
+      (int64_t{1} << 30))
+    return ISPA_ERR_INVALID_ARG;
+  AppendParams p;
+  memset(&p, 0, sizeof(p));
+  p.n_layers = n_layers;
+  p.n_frames = n_frames;
+  p.tokens_per_frame = r0.tokens_per_frame;
+  p.num_heads = r0.num_heads;
+  p.head_dim = r0.head_dim;
+  for (int l = 0; l < n_layers; ++l) {
+    const ispa_kv_ring& r = rings[l];
+    p.capacity_tokens[l] = r.capacity_frames * r.tokens_per_frame;
+    for (int i = 0; i < n_frames; ++i) p.slot[l][i] = slot_of(&r, r.frames_written + i);
+    p.k_src[l] = k_new[l];
+    p.v_src[l] = v_new[l];
+    p.k_dst[l] = r.k;
+    p.v_dst[l] = r.v;
+  }
+  if (launch_append(p, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  for (int l = 0; l < n_layers; ++l) rings[l].frames_written += n_frames;
+  return ISPA_OK;
+}
+
+ispa_status ispa_kv_append(ispa_kv_ring* ring, const void* k_new, const void* v_new,
+                           int32_t n_frames, ispa_stream stream) {
+  if (!ring) return ISPA_ERR_INVALID_ARG;
+  const void* k[1] = {k_new};
+  const void* v[1] = {v_new};
+  return ispa_kv_append_layers(ring, 1, k, v, n_frames, stream);
+}
+
+ispa_status ispa_attn_full(const ispa_kv_ring* ring, const void* q, const void* k_cur,
+                           const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
+                           ispa_stream stream) {
+  return attn_common(MODE_FULL, ring, ispa_window{0, 0}, q, k_cur, v_cur, n_q, scale, out, nullptr,
+                     lse, nullptr, nullptr, stream);
+}
+
+ispa_status ispa_attn_local(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                            const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                            void* out, float* lse, ispa_stream stream) {
+  return attn_common(MODE_LOCAL, ring, win, q, k_cur, v_cur, n_q, scale, out, nullptr, lse, nullptr,
+                     nullptr, stream);
+}
+
+size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q) {
+  if (num_heads <= 0 || n_q <= 0) return 0;
+  return static_cast<size_t>(num_heads) * n_q * sizeof(float);
+}
+
+ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                           const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                           void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                           float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                           ispa_stream stream) {
+  if (!ring || !disc || !disc_sq_sum) return ISPA_ERR_INVALID_ARG;
+  const size_t need = ispa_attn_dual_workspace_size(ring->num_heads, n_q);
+  if (need == 0) return ISPA_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
+  float* part = static_cast<float*>(workspace);
+  const ispa_status st = attn_common(MODE_DUAL, ring, win, q, k_cur, v_cur, n_q, scale, a_full,
+                                     a_loc, lse_full, lse_loc, part, stream);
+  if (st != ISPA_OK) return st;
+  if (launch_disc_reduce(part, ring->num_heads, n_q, disc, disc_sq_sum, stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+size_t ispa_ls_state_bytes(int32_t dim) {
+  if (dim <= 0) return 0;
+  return 4ull * dim * dim * sizeof(float);
+}
+
+ispa_status ispa_ls_state_reset(ispa_ls_state* st, ispa_stream stream) {
+  if (!st || st->dim <= 0 || !aligned16(st->gram)) return ISPA_ERR_INVALID_ARG;
+  if (cudaMemsetAsync(st->gram, 0, ispa_ls_state_bytes(st->dim), stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  st->n_tokens = 0;
+  return ISPA_OK;
+}
+
+size_t ispa_ls_accumulate_workspace_size(int32_t dim, int64_t T) {
+  if (dim <= 0 || T <= 0) return 0;
+  return ls_accumulate_ws_bytes(dim, T);
+}
+
+ispa_status ispa_ls_accumulate(ispa_ls_state* st, const void* a_loc, const void* a_full, int64_t T,
+                               void* workspace, size_t ws_bytes, ispa_stream stream) {
+  if (!st || st->dim <= 0 || T <= 0 || T > INT32_MAX || !aligned16(st->gram) || !aligned16(a_loc) ||
+      !aligned16(a_full))
+    return ISPA_ERR_INVALID_ARG;
+  if (st->dim % 128 != 0) return ISPA_ERR_UNSUPPORTED;
+  const size_t need = ls_accumulate_ws_bytes(st->dim, T);
+  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
+  int* status = device_status_ptr();
+  if (!status) return ISPA_ERR_CUDA;
+  if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, st->gram, status, g_wait_limit,
+                           stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  st->n_tokens += T;
+  return ISPA_OK;
+}
+
+size_t ispa_ls_solve_workspace_size(int32_t dim, int32_t d_out) {
+  if (dim <= 0 || d_out <= 0) return 0;
+  return ls_solve_ws_bytes(dim, d_out);
+}
+
+ispa_status ispa_ls_solve(const ispa_ls_state* st, const float* W, int32_t d_out, double lambda,
+                          float* dW, double* eps_out, void* workspace, size_t ws_bytes,
+                          ispa_stream stream) {
+  if (!st || st->dim <= 0 || d_out <= 0 || !aligned16(st->gram) || !aligned16(W) || !aligned16(dW))
+    return ISPA_ERR_INVALID_ARG;
+  if (!(lambda >= 0.0) || !isfinite(lambda)) return ISPA_ERR_INVALID_ARG;
+  const size_t need = ls_solve_ws_bytes(st->dim, d_out);
+  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
+  return run_ls_solve(st->dim, st->gram, W, d_out, lambda, dW, eps_out, workspace, stream);
+}
+
+}  // extern "C"

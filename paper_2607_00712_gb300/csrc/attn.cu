@@ -1,0 +1,466 @@
+// Chunk-step attention against the KV ring on sm_103a (tcgen05 + TMEM + TMA).
+//
+// One kernel serves the three modes of ISPA's attention:
+//   * F-layer (Eq. 3): keys = every resident past frame plus the chunk;
+//   * L-layer (Sec. 3.3, Eq. 7): keys = sink + recent window + chunk;
+//   * dual warmup (Sec. 3.1 phase 1, Sec. 3.4): the local segments are visited
+//     first; after the last local tile the running online-softmax state
+//     (O, m, l) is snapshotted as A_loc, and the same state keeps absorbing the
+//     history tiles to give A_full.  This is the LSE fusion of Eq. 11-12
+//     carried out inside one pass: the history branch's (O, LSE) is never
+//     materialised, every key is visited once, and the fusion costs one
+//     extra read of O from TMEM per row.
+//
+// Tensor maps: the ring as (d, cap*P, H) and the chunk tensors q/k_cur/v_cur
+// as (d, H, n_q), boxes of 64 x 128 rows x 1 head with 128-byte swizzle, which
+// is the K-major (Q, K) and MN-major (V) UMMA operand layout.
+// CTA = one head x one tile of 128 queries.  Warp roles:
+//   warps 0-3  softmax: thread t of warp w owns query row 32w+t (TMEM lane);
+//   warp 4     TMA producer (Q once, then K/V tiles into staged rings);
+//   warp 5     TMEM allocator and UMMA issuer.
+// TMEM columns: S0 [0,128) S1 [128,256) O [256,256+d) P0 [384,448) P1 [448,512).
+// Per key tile j: S_j = Q K_j^T (SS-UMMA, fp32 in TMEM) -> softmax warps read
+// S_j, update the row max (lazy rescale of O only when the max grows by more
+// than 2^8), write P_j = exp2(.) as bf16 into TMEM -> O += P_j V_j (TS-UMMA:
+// A operand read from TMEM).  S is double buffered so S_{j+1} runs on the
+// tensor cores while the softmax warps work on S_j.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ispa {
+
+namespace {
+
+constexpr int BM = 128;       // queries per CTA
+constexpr int BN = 128;       // keys per tile
+constexpr int NTHREADS = 192;
+constexpr int WARP_TMA = 4;
+constexpr int WARP_MMA = 5;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr float RESCALE_THRESHOLD = 8.0f;  // log2 units
+constexpr uint64_t DRAIN_LIMIT_NS = 200ull * 1000 * 1000;
+
+template <int HD>
+struct Cfg {
+  static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per tile row
+  static constexpr int BOX = 128 * 128;         // [128 rows][64 bf16] = 16 KB
+  static constexpr int TILE = NBOX * BOX;       // one Q, K or V tile
+  static constexpr int KST = HD == 128 ? 3 : 4;  // K stages
+  static constexpr int VST = HD == 128 ? 2 : 4;  // V stages
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = TILE;
+  static constexpr int OFF_V = OFF_K + KST * TILE;
+  static constexpr int OFF_BAR = OFF_V + VST * TILE;
+  static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
+  static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16 + 1024;  // + tmem slot/abort + alignment
+  static constexpr uint32_t COL_S0 = 0, COL_O = 256, COL_P0 = 384;
+  static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
+  static constexpr uint32_t IDESC_PV = idesc_bf16(BM, HD, false, true);
+};
+
+struct Bars {
+  uint32_t q_full, k_full0, k_empty0, v_full0, v_empty0, s_full0, p_full0, o_done0, drain;
+};
+
+__device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& off) {
+  off += BN;
+  if (off >= p.seg[seg].count) {
+    ++seg;
+    off = 0;
+  }
+}
+
+// Round 32 consecutive fp32 values (times inv) to bf16 pairs.
+__device__ __forceinline__ void pack_row32(const uint32_t* r, float inv, uint32_t* pk) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k)
+    pk[k] = pack_bf16x2(__uint_as_float(r[2 * k]) * inv, __uint_as_float(r[2 * k + 1]) * inv);
+}
+
+__device__ __forceinline__ void store_pk16(__nv_bfloat16* dst, const uint32_t* pk) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+}
+
+}  // namespace
+
+template <int HD>
+__global__ void __launch_bounds__(NTHREADS, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kr,
+                const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_kc,
+                const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
+  using C = Cfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int q_tile = blockIdx.x;
+  const int head = blockIdx.y;
+  const int q0 = q_tile * BM;
+
+  Bars b;
+  {
+    const uint32_t b0 = smem_u32(bar_mem);
+    b.q_full = b0;
+    b.k_full0 = b0 + 8 * 1;
+    b.k_empty0 = b.k_full0 + 8 * C::KST;
+    b.v_full0 = b.k_empty0 + 8 * C::KST;
+    b.v_empty0 = b.v_full0 + 8 * C::VST;
+    b.s_full0 = b.v_empty0 + 8 * C::VST;
+    b.p_full0 = b.s_full0 + 16;
+    b.o_done0 = b.p_full0 + 16;
+    b.drain = b.o_done0 + 16;
+  }
+
+  if (threadIdx.x == 0) {
+    mbar_init(b.q_full, 1);
+    for (int i = 0; i < C::KST; ++i) {
+      mbar_init(b.k_full0 + 8 * i, 1);
+      mbar_init(b.k_empty0 + 8 * i, 1);
+    }
+    for (int i = 0; i < C::VST; ++i) {
+      mbar_init(b.v_full0 + 8 * i, 1);
+      mbar_init(b.v_empty0 + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b.s_full0 + 8 * i, 1);
+      mbar_init(b.p_full0 + 8 * i, BM);
+      mbar_init(b.o_done0 + 8 * i, 1);
+    }
+    mbar_init(b.drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == WARP_MMA) {
+    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+    tmem_relinquish();
+  }
+  if (warp == WARP_TMA && lane == 0) {
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kr);
+    tma_prefetch_desc(&tm_vr);
+    tma_prefetch_desc(&tm_kc);
+    tma_prefetch_desc(&tm_vc);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
+  const int n_tiles = p.n_tiles;
+
+  if (warp == WARP_TMA) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint32_t sQ = sbase + C::OFF_Q;
+      mbar_arrive_expect_tx(b.q_full, C::TILE);
+#pragma unroll
+      for (int x = 0; x < C::NBOX; ++x) tma_load_3d(sQ + x * C::BOX, &tm_q, b.q_full, 64 * x, head, q0);
+      int seg = 0, off = 0;
+      int nk = 0, nv = 0;  // K and V tiles issued
+      for (int j = 0; j < n_tiles; ++j) {
+        const bool chunk = p.seg[seg].src != 0;
+        const int row = p.seg[seg].start + off;
+        const int ks = j % C::KST, vs = j % C::VST;
+        if (!mbar_wait(b.k_empty0 + 8 * ks, ((j / C::KST) & 1) ^ 1, wc)) break;
+        mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::TILE);
+        const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
+#pragma unroll
+        for (int x = 0; x < C::NBOX; ++x) {
+          if (chunk) tma_load_3d(sK + x * C::BOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
+          else tma_load_3d(sK + x * C::BOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
+        }
+        nk = j + 1;
+        if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc)) break;
+        mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::TILE);
+        const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
+#pragma unroll
+        for (int x = 0; x < C::NBOX; ++x) {
+          if (chunk) tma_load_3d(sV + x * C::BOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
+          else tma_load_3d(sV + x * C::BOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
+        }
+        nv = j + 1;
+        next_tile(p, seg, off);
+      }
+      // Every load issued must have landed before the CTA may exit.  Older tiles of
+      // a stage completed before the stage was refilled, so the last KST (VST) suffice.
+      mbar_wait_drain(b.q_full, 0, DRAIN_LIMIT_NS);
+      for (int t = nk > C::KST ? nk - C::KST : 0; t < nk; ++t)
+        mbar_wait_drain(b.k_full0 + 8 * (t % C::KST), (t / C::KST) & 1, DRAIN_LIMIT_NS);
+      for (int t = nv > C::VST ? nv - C::VST : 0; t < nv; ++t)
+        mbar_wait_drain(b.v_full0 + 8 * (t % C::VST), (t / C::VST) & 1, DRAIN_LIMIT_NS);
+    }
+    __syncwarp();
+  } else if (warp == WARP_MMA) {
+    // ------------------------------------------------------------ UMMA issuer
+    if (lane == 0) {
+      const uint32_t sQ = sbase + C::OFF_Q;
+      bool ok = mbar_wait(b.q_full, 0, wc);
+      tc_fence_after();
+      auto issue_s = [&](int j) -> bool {
+        const int ks = j % C::KST;
+        if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc)) return false;
+        tc_fence_after();
+        const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
+        const uint32_t d = tmem + C::COL_S0 + (j & 1) * 128;
+#pragma unroll
+        for (int k = 0; k < HD / 16; ++k) {
+          const uint32_t koff = (k >> 2) * C::BOX + (k & 3) * 32;
+          umma_ss(d, sw128_desc(sQ + koff, 16, 1024), sw128_desc(sK + koff, 16, 1024), C::IDESC_QK,
+                  k > 0 ? 1u : 0u);
+        }
+        tc_commit(b.s_full0 + 8 * (j & 1));
+        tc_commit(b.k_empty0 + 8 * ks);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      if (ok && n_tiles > 1) ok = issue_s(1);
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int vs = j % C::VST;
+        if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc)) break;
+        if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc)) break;
+        tc_fence_after();
+        const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
+        const uint32_t a = tmem + C::COL_P0 + (j & 1) * 64;
+#pragma unroll
+        for (int k = 0; k < BN / 16; ++k) {
+          umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::BOX, 1024), C::IDESC_PV,
+                  (j > 0 || k > 0) ? 1u : 0u);
+        }
+        tc_commit(b.o_done0 + 8 * (j & 1));
+        tc_commit(b.v_empty0 + 8 * vs);
+        if (j + 2 < n_tiles) ok = issue_s(j + 2);
+      }
+      // All UMMAs must have finished before TMEM is released.
+      tc_commit(b.drain);
+      mbar_wait_drain(b.drain, 0, DRAIN_LIMIT_NS);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax warps
+    const int row = warp * 32 + lane;
+    const int qrow = q0 + row;
+    const bool row_ok = qrow < p.n_q;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const int D = p.num_heads * HD;
+    const float sl2 = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    int seg = 0, off = 0;
+    bool ok = true;
+
+    auto warp_ok = [&](bool v) { return __all_sync(0xffffffffu, v); };
+
+    auto emit = [&](__nv_bfloat16* dst, float* lse_dst, bool with_disc) {
+      // O / l of this row -> bf16 global; optional LSE; optional discrepancy partial
+      // sum_d (A_full - A_loc)^2 of this head, taken on the stored bf16 values.
+      const float inv = 1.f / l_run;
+      __nv_bfloat16* drow = dst + static_cast<size_t>(qrow) * D + head * HD;
+      const __nv_bfloat16* lrow = p.out_loc + static_cast<size_t>(qrow) * D + head * HD;
+      float sq = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(trow + C::COL_O + 32 * c, r);
+        tmem_wait_ld32(r);
+        if (row_ok) {
+          uint32_t pk[16];
+          pack_row32(r, inv, pk);
+          store_pk16(drow + 32 * c, pk);
+          if (with_disc) {
+            const uint4* l4 = reinterpret_cast<const uint4*>(lrow + 32 * c);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const uint4 v = l4[q];
+              const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const uint32_t f = pk[4 * q + e];
+                const float d0 = __uint_as_float(f << 16) - __uint_as_float(w[e] << 16);
+                const float d1 = __uint_as_float(f & 0xFFFF0000u) - __uint_as_float(w[e] & 0xFFFF0000u);
+                sq = fmaf(d0, d0, sq);
+                sq = fmaf(d1, d1, sq);
+              }
+            }
+          }
+        }
+      }
+      if (row_ok) {
+        if (lse_dst)
+          lse_dst[static_cast<size_t>(head) * p.n_q + qrow] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
+        if (with_disc) p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = sq;
+      }
+    };
+
+    for (int j = 0; j < n_tiles; ++j) {
+      const int sb = j & 1;
+      if (p.dual && j == p.n_local_tiles && j > 0) {
+        // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc));
+        if (!ok) break;
+        tc_fence_after();
+        emit(p.out_loc, p.lse_loc, false);
+      }
+      ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc));
+      if (!ok) break;
+      tc_fence_after();
+      const int valid = min(BN, p.seg[seg].count - off);
+      uint32_t s[BN];
+      tmem_ld32(trow + C::COL_S0 + sb * 128 + 0, s + 0);
+      tmem_ld32(trow + C::COL_S0 + sb * 128 + 32, s + 32);
+      tmem_ld32(trow + C::COL_S0 + sb * 128 + 64, s + 64);
+      tmem_ld32(trow + C::COL_S0 + sb * 128 + 96, s + 96);
+      tmem_wait_ld32(s + 0);
+      tmem_wait_ld32(s + 32);
+      tmem_wait_ld32(s + 64);
+      tmem_wait_ld32(s + 96);
+      if (valid < BN) {
+#pragma unroll
+        for (int i = 0; i < BN; ++i)
+          if (i >= valid) s[i] = __float_as_uint(-INFINITY);
+      }
+      float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < BN; i += 4) {
+        mx0 = fmaxf(mx0, __uint_as_float(s[i + 0]));
+        mx1 = fmaxf(mx1, __uint_as_float(s[i + 1]));
+        mx2 = fmaxf(mx2, __uint_as_float(s[i + 2]));
+        mx3 = fmaxf(mx3, __uint_as_float(s[i + 3]));
+      }
+      const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+      if (j == 0) {
+        m_run = m_tile;
+      } else if (m_tile > m_run + RESCALE_THRESHOLD) {
+        // Lazy rescale: O holds PV of tiles 0..j-1 once PV_{j-1} has completed.
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc));
+        if (!ok) break;
+        tc_fence_after();
+        const float alpha = ex2_approx(m_run - m_tile);
+        l_run *= alpha;
+#pragma unroll 1
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(trow + C::COL_O + 32 * c, r);
+          tmem_wait_ld32(r);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+          tmem_st32(trow + C::COL_O + 32 * c, r);
+        }
+        tmem_wait_st();
+        m_run = m_tile;
+      }
+      // P_j goes to TMEM buffer sb, last read by PV_{j-2}.
+      if (j >= 2) {
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc));
+        if (!ok) break;
+        tc_fence_after();
+      }
+      const float neg_m = -m_run;
+      float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const float e0 = ex2_approx(fmaf(__uint_as_float(s[32 * c + 2 * k]), sl2, neg_m));
+          const float e1 = ex2_approx(fmaf(__uint_as_float(s[32 * c + 2 * k + 1]), sl2, neg_m));
+          rs0 += e0;
+          rs1 += e1;
+          pk[k] = pack_bf16x2(e0, e1);
+        }
+        tmem_st16(trow + C::COL_P0 + sb * 64 + 16 * c, pk);
+      }
+      l_run += rs0 + rs1;
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(b.p_full0 + 8 * sb);
+      next_tile(p, seg, off);
+    }
+    if (ok) {
+      const int jl = n_tiles - 1;
+      ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc));
+      if (ok) {
+        tc_fence_after();
+        if (p.dual && p.n_local_tiles >= n_tiles) emit(p.out_loc, p.lse_loc, false);
+        emit(p.out, p.lse, p.dual != 0);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == WARP_MMA) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+template <int HD>
+static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, const CUtensorMap* tvr,
+                             const CUtensorMap* tkc, const CUtensorMap* tvc, const AttnParams& p,
+                             cudaStream_t s) {
+  using C = Cfg<HD>;
+  static bool attr_done[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_done[dev] = true;
+  }
+  dim3 grid((p.n_q + BM - 1) / BM, p.num_heads);
+  attn_kernel<HD><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attention(int head_dim, const CUtensorMap* tq, const CUtensorMap* tkr,
+                             const CUtensorMap* tvr, const CUtensorMap* tkc,
+                             const CUtensorMap* tvc, const AttnParams& p, cudaStream_t s) {
+  if (head_dim == 128) return launch_hd<128>(tq, tkr, tvr, tkc, tvc, p, s);
+  if (head_dim == 64) return launch_hd<64>(tq, tkr, tvr, tkc, tvc, p, s);
+  return cudaErrorInvalidValue;
+}
+
+// ------------------------------------------------------------ discrepancy reduction
+// disc[t] = sqrt(sum_h part[h][t]);  *disc_sq_sum += sum over the block's tokens.
+__global__ void __launch_bounds__(256) disc_reduce_kernel(const float* __restrict__ part, int H,
+                                                          int n_q, float* __restrict__ disc,
+                                                          float* __restrict__ disc_sq_sum) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  float v = 0.f;
+  if (t < n_q) {
+    for (int h = 0; h < H; ++h) v += part[static_cast<size_t>(h) * n_q + t];
+    disc[t] = sqrtf(v);
+  }
+  __shared__ float red[8];
+  float w = v;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = w;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    w = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
+    if (threadIdx.x == 0) atomicAdd(disc_sq_sum, w);
+  }
+}
+
+cudaError_t launch_disc_reduce(const float* part, int32_t H, int32_t n_q, float* disc,
+                               float* disc_sq_sum, cudaStream_t s) {
+  if (n_q <= 0) return cudaSuccess;
+  disc_reduce_kernel<<<(n_q + 255) / 256, 256, 0, s>>>(part, H, n_q, disc, disc_sq_sum);
+  return cudaGetLastError();
+}
+
+}  // namespace ispa

@@ -1,0 +1,315 @@
+// Normal-equation sums of the least-squares absorption (Sec. 3.2, Eq. 5):
+//   G += A_loc^T A_loc,  X += A_loc^T Delta,  S += Delta^T Delta,
+// with Delta = A_full - A_loc, on the tensor cores (tcgen05, fp32 in TMEM).
+//
+// Step 1 (split_kernel, HBM-bound): Delta is formed exactly in fp32 from the
+// two bf16 inputs and stored as a bf16 pair hi = bf16(Delta),
+// lo = bf16(Delta - hi), so hi + lo carries Delta to ~2^-16 relative.
+// Step 2 (gram_kernel): every output tile 128 x BN of the upper blocks is a
+// contraction over tokens, the token axis being the UMMA K dimension:
+//   G tile: a^T a;   X tile: a^T hi + a^T lo;   S tile: hi^T hi + hi^T lo + lo^T hi
+// (the lo^T lo term is below fp32 resolution and dropped).  Both operands
+// are token-major [T][D] in HBM, i.e. MN-major for the UMMA, staged by TMA in
+// 64-token x 64-feature boxes with 128-byte swizzle.  Tokens are split across
+// CTAs (blockIdx.y) and each CTA adds its partial tile into the fp32 state
+// with vector atomics.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ispa {
+
+namespace {
+
+constexpr int GM = 128;        // output rows per tile
+constexpr int GK = 64;         // tokens per stage
+constexpr int GST = 4;         // pipeline stages
+constexpr int G_THREADS = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr uint64_t G_DRAIN_NS = 200ull * 1000 * 1000;
+
+template <int BN>
+struct GCfg {
+  static constexpr int BOX = GK * 128;            // 64 tokens x 64 features bf16 = 8 KB
+  static constexpr int A_BYTES = (GM / 64) * BOX;  // 16 KB
+  static constexpr int B_BYTES = (BN / 64) * BOX;
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int OFF_BAR = GST * STAGE;
+  static constexpr int SMEM = OFF_BAR + (2 * GST + 2) * 8 + 16 + 1024;
+  static constexpr uint32_t IDESC = idesc_bf16(GM, BN, true, true);
+  static constexpr uint32_t TMEM_COLS = BN;  // 128 or 256, both powers of two
+};
+
+// Operand sources of the passes of each block type: 0 = A_loc, 1 = hi, 2 = lo.
+struct Pass {
+  int8_t a, b;
+};
+__constant__ Pass kPasses[3][3] = {
+    {{0, 0}, {0, 0}, {0, 0}},  // G: one pass
+    {{0, 1}, {0, 2}, {0, 0}},  // X: two passes
+    {{1, 1}, {1, 2}, {2, 1}},  // S: three passes
+};
+__constant__ int kNumPasses[3] = {1, 2, 3};
+
+struct GramParams {
+  int32_t D;
+  int32_t T;
+  int32_t n_ktiles;   // ceil(T / GK)
+  int32_t kt_per_split;
+  float* gram;        // [2D][2D]
+  int* status;
+  uint64_t wait_limit_ns;
+};
+
+// Decode blockIdx.x into (kind, row block, col block).  Items: upper G tiles,
+// then all X tiles, then upper S tiles.
+template <int BN>
+__device__ __forceinline__ void decode_tile(int item, int D, int& kind, int& bi, int& bj) {
+  const int RB = D / GM, CB = D / BN;
+  int n_upper = 0;
+  for (int r = 0; r < RB; ++r) n_upper += CB - (r * GM) / BN;
+  kind = 0;
+  if (item >= n_upper) {
+    item -= n_upper;
+    if (item < RB * CB) {
+      kind = 1;
+      bi = item / CB;
+      bj = item % CB;
+      return;
+    }
+    item -= RB * CB;
+    kind = 2;
+  }
+  for (int r = 0; r < RB; ++r) {
+    const int c0 = (r * GM) / BN;
+    const int n = CB - c0;
+    if (item < n) {
+      bi = r;
+      bj = c0 + item;
+      return;
+    }
+    item -= n;
+  }
+  bi = bj = 0;
+}
+
+}  // namespace
+
+// Delta = a_full - a_loc (exact in fp32), hi = bf16(Delta), lo = bf16(Delta - hi).
+__global__ void __launch_bounds__(256) split_kernel(const uint4* __restrict__ a_loc,
+                                                    const uint4* __restrict__ a_full,
+                                                    uint4* __restrict__ hi, uint4* __restrict__ lo,
+                                                    int64_t n_words) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
+    const uint4 a = a_loc[i], f = a_full[i];
+    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float d0 = __uint_as_float(fw[e] << 16) - __uint_as_float(aw[e] << 16);
+      const float d1 = __uint_as_float(fw[e] & 0xFFFF0000u) - __uint_as_float(aw[e] & 0xFFFF0000u);
+      const uint32_t h = pack_bf16x2(d0, d1);
+      const float h0 = __uint_as_float(h << 16), h1 = __uint_as_float(h & 0xFFFF0000u);
+      hw[e] = h;
+      lw[e] = pack_bf16x2(d0 - h0, d1 - h1);
+    }
+    hi[i] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    lo[i] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(G_THREADS, 1)
+    gram_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_hi,
+                const __grid_constant__ CUtensorMap tm_lo, const GramParams p) {
+  using C = GCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * GST + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * GST, acc_bar = empty0 + 8 * GST,
+                 drain_bar = acc_bar + 8;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int kind, bi, bj;
+  decode_tile<BN>(blockIdx.x, p.D, kind, bi, bj);
+  const int kt0 = blockIdx.y * p.kt_per_split;
+  const int kt1 = min(p.n_ktiles, kt0 + p.kt_per_split);
+  const int n_kt = kt1 - kt0;
+  const int n_pass = kNumPasses[kind];
+  const int total_steps = n_pass * n_kt;
+  // feature offsets inside the [T][D] operands
+  const int fa = bi * GM;   // rows of the output tile = features of operand A
+  const int fb = bj * BN;   // cols of the output tile = features of operand B
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < GST; ++i) {
+      mbar_init(full0 + 8 * i, 1);
+      mbar_init(empty0 + 8 * i, 1);
+    }
+    mbar_init(acc_bar, 1);
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
+
+  if (warp == 0) {
+    if (lane == 0 && total_steps > 0) {
+      const CUtensorMap* maps[3] = {&tm_a, &tm_hi, &tm_lo};
+      int issued = 0;
+      for (int s = 0; s < total_steps; ++s) {
+        const int pass = s / n_kt;
+        const int tok = (kt0 + s % n_kt) * GK;
+        const int st = s % GST;
+        if (!mbar_wait(empty0 + 8 * st, ((s / GST) & 1) ^ 1, wc)) break;
+        mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
+        const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
+        const CUtensorMap* ma = maps[kPasses[kind][pass].a];
+        const CUtensorMap* mb = maps[kPasses[kind][pass].b];
+#pragma unroll
+        for (int x = 0; x < GM / 64; ++x) tma_load_2d(sa + x * C::BOX, ma, full0 + 8 * st, fa + 64 * x, tok);
+#pragma unroll
+        for (int x = 0; x < BN / 64; ++x) tma_load_2d(sb + x * C::BOX, mb, full0 + 8 * st, fb + 64 * x, tok);
+        issued = s + 1;
+      }
+      for (int s = issued > GST ? issued - GST : 0; s < issued; ++s)
+        mbar_wait_drain(full0 + 8 * (s % GST), (s / GST) & 1, G_DRAIN_NS);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && total_steps > 0) {
+      bool ok = true;
+      for (int s = 0; s < total_steps; ++s) {
+        const int st = s % GST;
+        if (!mbar_wait(full0 + 8 * st, (s / GST) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
+#pragma unroll
+        for (int k = 0; k < GK / 16; ++k)
+          umma_ss(tmem, sw128_desc(sa + k * 2048, C::BOX, 1024), sw128_desc(sb + k * 2048, C::BOX, 1024),
+                  C::IDESC, (s > 0 || k > 0) ? 1u : 0u);
+        tc_commit(empty0 + 8 * st);
+      }
+      if (ok) tc_commit(acc_bar);
+      tc_commit(drain_bar);
+      mbar_wait_drain(drain_bar, 0, G_DRAIN_NS);
+    }
+    __syncwarp();
+  } else if (total_steps > 0) {
+    // epilogue: warp w reads TMEM lanes 32*(w%4) .. +31 = output rows
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, wc));
+    if (ok) {
+      tc_fence_after();
+      const int D = p.D;
+      const int row0 = (kind == 2 ? D : 0) + fa;
+      const int col0 = (kind == 0 ? 0 : D) + fb;
+      float* grow = p.gram + static_cast<size_t>(row0 + r) * (2 * D) + col0;
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(taddr + 32 * c, v);
+        tmem_wait_ld32(v);
+        float4* g4 = reinterpret_cast<float4*>(grow + 32 * c);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          atomicAdd(g4 + q, make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                        __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3])));
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+size_t ls_accumulate_ws_bytes(int32_t D, int64_t T) {
+  // hi and lo, each bf16 [T][D], 256-byte aligned
+  const size_t one = (static_cast<size_t>(T) * D * 2 + 255) & ~static_cast<size_t>(255);
+  return 2 * one;
+}
+
+template <int BN>
+static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
+                               float* gram, int* status, uint64_t wait_limit_ns, cudaStream_t s) {
+  using C = GCfg<BN>;
+  static bool attr_done[64] = {};
+  int dev = 0, sms = 152;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(gram_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_done[dev] = true;
+  }
+  CUtensorMap ta, th, tl;
+  if (!encode_tmap_2d(&ta, a_loc, D, T, static_cast<uint64_t>(D) * 2, 64, GK) ||
+      !encode_tmap_2d(&th, hi, D, T, static_cast<uint64_t>(D) * 2, 64, GK) ||
+      !encode_tmap_2d(&tl, lo, D, T, static_cast<uint64_t>(D) * 2, 64, GK))
+    return cudaErrorInvalidValue;
+  const int RB = D / GM, CB = D / BN;
+  int n_upper = 0;
+  for (int r = 0; r < RB; ++r) n_upper += CB - (r * GM) / BN;
+  const int n_items = 2 * n_upper + RB * CB;
+  GramParams p;
+  p.D = D;
+  p.T = static_cast<int32_t>(T);
+  p.n_ktiles = static_cast<int32_t>((T + GK - 1) / GK);
+  // token splits: aim at >= 3 CTAs per SM over all items, at least 8 token tiles each
+  int splits = (3 * sms + n_items - 1) / n_items;
+  splits = max(1, min(splits, p.n_ktiles / 8 > 0 ? p.n_ktiles / 8 : 1));
+  p.kt_per_split = (p.n_ktiles + splits - 1) / splits;
+  splits = (p.n_ktiles + p.kt_per_split - 1) / p.kt_per_split;
+  p.gram = gram;
+  p.status = status;
+  p.wait_limit_ns = wait_limit_ns;
+  dim3 grid(n_items, splits);
+  gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(ta, th, tl, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full, void* ws,
+                                 float* gram, int* status, uint64_t wait_limit_ns, cudaStream_t s) {
+  const size_t one = ls_accumulate_ws_bytes(D, T) / 2;
+  uint8_t* hi = static_cast<uint8_t*>(ws);
+  uint8_t* lo = hi + one;
+  const int64_t n_words = static_cast<int64_t>(T) * D / 8;
+  int dev = 0, sms = 152;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t blocks = (n_words + 255) / 256;
+  if (blocks > static_cast<int64_t>(sms) * 8) blocks = static_cast<int64_t>(sms) * 8;
+  split_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+      static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), reinterpret_cast<uint4*>(hi),
+      reinterpret_cast<uint4*>(lo), n_words);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (D % 256 == 0) return launch_gram<256>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, s);
+  return launch_gram<128>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, s);
+}
+
+}  // namespace ispa

@@ -1,0 +1,94 @@
+// Internal declarations shared by the translation units of libispa (host side).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/ispa.h"
+
+namespace ispa {
+
+// ------------------------------------------------------------ attention
+// One contiguous run of keys.  src 0 = the KV ring ([H][cap*P][d]), src 1 = the
+// chunk's own k_cur/v_cur ([n_q][H][d]).  start/count are token rows.
+struct AttnSeg {
+  int32_t src;
+  int32_t start;
+  int32_t count;
+  int32_t pad;
+};
+
+constexpr int kMaxSegs = 8;
+
+struct AttnParams {
+  int32_t n_q;
+  int32_t num_heads;
+  int32_t n_seg;           // segments in seg[]
+  int32_t n_tiles;         // total key tiles over all segments
+  int32_t n_local_tiles;   // dual: tiles of the local set (they come first)
+  int32_t dual;            // 1 = emit A_loc snapshot and discrepancy partials
+  float scale_log2;        // softmax scale * log2(e)
+  int32_t pad;
+  uint64_t wait_limit_ns;  // bounded-wait limit
+  AttnSeg seg[kMaxSegs];
+  __nv_bfloat16* out;      // [n_q][H*d]  (A_full in dual mode)
+  __nv_bfloat16* out_loc;  // [n_q][H*d]  dual only
+  float* lse;              // [H][n_q] or null
+  float* lse_loc;          // [H][n_q] or null (dual)
+  float* disc_part;        // [H][n_q] per-head sum of squared discrepancy (dual)
+  int* status;             // library status word
+};
+
+// Launch the attention kernel.  tensor maps are encoded by the caller.
+cudaError_t launch_attention(int head_dim, const CUtensorMap* tm_q, const CUtensorMap* tm_kr,
+                             const CUtensorMap* tm_vr, const CUtensorMap* tm_kc,
+                             const CUtensorMap* tm_vc, const AttnParams& p, cudaStream_t s);
+// disc[t] = sqrt(sum_h part[h][t]); *disc_sq_sum += sum_t sum_h part[h][t]
+cudaError_t launch_disc_reduce(const float* part, int32_t H, int32_t n_q, float* disc,
+                               float* disc_sq_sum, cudaStream_t s);
+
+// ------------------------------------------------------------ KV append
+constexpr int kMaxAppendFrames = 16;
+constexpr int kMaxAppendLayers = 64;
+
+struct AppendParams {
+  int32_t n_layers;
+  int32_t n_frames;
+  int32_t tokens_per_frame;
+  int32_t num_heads;
+  int32_t head_dim;
+  int32_t pad;
+  int32_t capacity_tokens[kMaxAppendLayers];           // capacity_frames * P of each layer's ring
+  int32_t slot[kMaxAppendLayers][kMaxAppendFrames];    // ring slot of each appended frame
+  const void* k_src[kMaxAppendLayers];
+  const void* v_src[kMaxAppendLayers];
+  void* k_dst[kMaxAppendLayers];
+  void* v_dst[kMaxAppendLayers];
+};
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+
+// ------------------------------------------------------------ least squares
+// Accumulate the upper blocks of [A | dlt]^T [A | dlt] into the fp32 state.
+cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full,
+                                 void* ws, float* gram, int* status, uint64_t wait_limit_ns,
+                                 cudaStream_t s);
+size_t ls_accumulate_ws_bytes(int32_t D, int64_t T);
+
+size_t ls_solve_ws_bytes(int32_t D, int32_t d_out);
+// Returns ISPA_OK, ISPA_ERR_NOT_SPD or ISPA_ERR_CUDA; synchronises the stream.
+ispa_status run_ls_solve(int32_t D, const float* gram, const float* W, int32_t d_out,
+                         double lambda, float* dW, double* eps_out, void* ws, cudaStream_t s);
+
+// ------------------------------------------------------------ misc
+int* device_status_ptr();  // library status word on the current device (nullptr on error)
+bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                    uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
+                    uint32_t b2);
+bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
+                    uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
+uint64_t wait_limit_ns();
+
+}  // namespace ispa

@@ -1,0 +1,170 @@
+"""GPU parity: chunk-step attention (full / local / dual) through the C-ABI vs the fp64 oracle.
+
+Tolerance (bf16 outputs, fp32 accumulation): max-abs <= 2e-2, mean-abs <= 2e-3.
+"""
+import math
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from gpu_helpers import Step, assert_close_attn  # noqa: E402
+from oracle import attention as at  # noqa: E402
+from paper_2607_00712_gb300 import abi  # noqa: E402
+from paper_2607_00712_gb300.device import Window, bf16_tensor, to_f32  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2607_00712_gb300.build import build_library
+    build_library()
+    abi.lib()
+
+
+def _run_full(st: Step, scale=0.0):
+    out = torch.empty(st.n_q, st.H * st.d, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(st.H, st.n_q, dtype=torch.float32, device="cuda")
+    abi.ispa_attn_full(st.ring.c, st.q, st.kc, st.vc, st.n_q, scale, out, lse)
+    torch.cuda.synchronize()
+    return to_f32(out).reshape(st.n_q, st.H, st.d), to_f32(lse)
+
+
+def _run_local(st: Step, win, scale=0.0):
+    out = torch.empty(st.n_q, st.H * st.d, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(st.H, st.n_q, dtype=torch.float32, device="cuda")
+    abi.ispa_attn_local(st.ring.c, Window(*win), st.q, st.kc, st.vc, st.n_q, scale, out, lse)
+    torch.cuda.synchronize()
+    return to_f32(out).reshape(st.n_q, st.H, st.d), to_f32(lse)
+
+
+def _run_dual(st: Step, win, scale=0.0, disc_sum=None):
+    D = st.H * st.d
+    a_full = torch.empty(st.n_q, D, dtype=torch.bfloat16, device="cuda")
+    a_loc = torch.empty(st.n_q, D, dtype=torch.bfloat16, device="cuda")
+    disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+    if disc_sum is None:
+        disc_sum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    lf = torch.empty(st.H, st.n_q, dtype=torch.float32, device="cuda")
+    ll = torch.empty(st.H, st.n_q, dtype=torch.float32, device="cuda")
+    wsb = abi.ispa_attn_dual_workspace_size(st.H, st.n_q)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    abi.ispa_attn_dual(st.ring.c, Window(*win), st.q, st.kc, st.vc, st.n_q, scale, a_full, a_loc, disc,
+                       disc_sum, lf, ll, ws, wsb)
+    torch.cuda.synchronize()
+    return dict(a_full=to_f32(a_full).reshape(st.n_q, st.H, st.d), a_loc=to_f32(a_loc).reshape(st.n_q, st.H, st.d),
+                disc=to_f32(disc), disc_sum=float(disc_sum.item()), lse_full=to_f32(lf), lse_loc=to_f32(ll))
+
+
+def _check_all_modes(st: Step, win, scale=0.0):
+    args = st.oracle_args()
+    o, l = _run_full(st, scale)
+    ro, rl = at.attn_full(*args, scale=scale)
+    assert_close_attn(o, ro, "full")
+    assert np.abs(l - rl).max() < 2e-3
+    o, l = _run_local(st, win, scale)
+    ro, rl = at.attn_local(*args, *win, scale=scale)
+    assert_close_attn(o, ro, "local")
+    assert np.abs(l - rl).max() < 2e-3
+    g = _run_dual(st, win, scale)
+    r = at.attn_dual(*args, *win, scale=scale)
+    assert_close_attn(g["a_full"], r["a_full"], "dual a_full")
+    assert_close_attn(g["a_loc"], r["a_loc"], "dual a_loc")
+    assert np.abs(g["lse_full"] - r["lse_full"]).max() < 2e-3
+    assert np.abs(g["lse_loc"] - r["lse_loc"]).max() < 2e-3
+    # disc is the norm of the difference of the two stored bf16 outputs ...
+    d_own = np.sqrt(((g["a_full"].astype(np.float64) - g["a_loc"]) ** 2).reshape(st.n_q, -1).sum(1))
+    assert np.allclose(g["disc"], d_own, rtol=1e-5, atol=1e-6)
+    assert abs(g["disc_sum"] - float((d_own ** 2).sum())) <= 1e-4 * max(1.0, float((d_own ** 2).sum()))
+    # ... which is within the outputs' own error of the oracle's exact discrepancy
+    D = st.H * st.d
+    assert np.abs(g["disc"] - r["disc"]).max() <= 2 * 2e-2 * math.sqrt(D)
+    assert np.abs(g["disc"] - r["disc"]).mean() <= 2 * 2e-3 * math.sqrt(D)
+
+
+def test_config0_tiny():
+    # 2 heads, d = 64, 64 tokens/frame, chunk of 2 frames (128 queries), 4 cached frames
+    # (384 keys in the full set), window = chunk + 2 most recent frames.
+    st = Step(0, P=64, H=2, d=64, n_past=4, n_chunk_frames=2, capacity=4)
+    _check_all_modes(st, (0, 2))
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_ragged_tiles_and_ring_wrap(d):
+    # 100 tokens per frame (tiles straddle frames), 300 queries (ragged tail), a ring of 7
+    # frames with one pinned sink that has wrapped (12 frames written).
+    st = Step(1, P=100, H=3, d=d, n_past=12, n_chunk_frames=3, capacity=7, n_sink_pinned=1)
+    for win in [(1, 2), (0, 3), (1, 0), (1, 6)]:
+        _check_all_modes(st, win)
+
+
+def test_explicit_scale_and_single_frame_chunk():
+    st = Step(2, P=72, H=2, d=64, n_past=5, n_chunk_frames=1, capacity=8)
+    _check_all_modes(st, (0, 2), scale=0.21)
+
+
+def test_no_history():
+    # F = 0: every mode sees only the chunk.
+    st = Step(3, P=64, H=2, d=128, n_past=0, n_chunk_frames=2, capacity=4)
+    o_full, _ = _run_full(st)
+    o_loc, _ = _run_local(st, (0, 2))
+    assert np.array_equal(o_full, o_loc)
+    g = _run_dual(st, (0, 2))
+    assert np.array_equal(g["a_full"], g["a_loc"]) and np.all(g["disc"] == 0)
+
+
+def test_values_all_one():
+    st = Step(4, P=64, H=2, d=128, n_past=3, n_chunk_frames=2, capacity=4)
+    st.ring.v.fill_(1.0)
+    st.vc.fill_(1.0)
+    o, _ = _run_full(st)
+    assert np.all(o == 1.0)
+    o, _ = _run_local(st, (0, 1))
+    assert np.all(o == 1.0)
+
+
+def test_empty_history_dual_is_exact():
+    # window covers the whole cache: hist is empty, A_full == A_loc bit for bit, disc == 0
+    st = Step(5, P=96, H=2, d=128, n_past=4, n_chunk_frames=2, capacity=6)
+    g = _run_dual(st, (0, 4))
+    assert np.array_equal(g["a_full"], g["a_loc"])
+    assert np.all(g["disc"] == 0) and g["disc_sum"] == 0.0
+    # and local over that window matches full within tolerance
+    o_full, _ = _run_full(st)
+    o_loc, _ = _run_local(st, (0, 4))
+    assert_close_attn(o_loc, o_full, "window covering cache")
+
+
+def test_disc_sum_accumulates():
+    st = Step(6, P=64, H=2, d=64, n_past=4, n_chunk_frames=2, capacity=4)
+    acc = torch.zeros(1, dtype=torch.float32, device="cuda")
+    g1 = _run_dual(st, (0, 1), disc_sum=acc)
+    g2 = _run_dual(st, (0, 1), disc_sum=acc)
+    one = float((g1["disc"].astype(np.float64) ** 2).sum())
+    assert abs(g2["disc_sum"] - 2 * one) <= 1e-4 * 2 * one
+
+
+def test_config1_sampled_rows():
+    # The 1.3B-shaped chunk step the bench times: 12 heads x 128, 1560 tokens/frame, 4680 queries,
+    # 18 cached frames (28080 keys + 4680 chunk keys), window = chunk + 6 frames.  Rows are
+    # independent, so the oracle on sampled rows is exact for those rows.
+    st = Step(7, P=1560, H=12, d=128, n_past=18, n_chunk_frames=3, capacity=18)
+    rng = np.random.default_rng(0)
+    rows = np.unique(np.concatenate([[0, 127, 128, 4607, 4608, 4679], rng.choice(4680, 58, replace=False)]))
+    args = st.oracle_args()
+    o, l = _run_full(st)
+    ro, rl = at.attn_full(*args, rows=rows)
+    assert_close_attn(o[rows], ro, "config1 full")
+    assert np.abs(l[:, rows] - rl).max() < 2e-3
+    o, _ = _run_local(st, (0, 6))
+    ro, _ = at.attn_local(*args, 0, 6, rows=rows)
+    assert_close_attn(o[rows], ro, "config1 local")
+    g = _run_dual(st, (0, 6))
+    r = at.attn_dual(*args, 0, 6, rows=rows)
+    assert_close_attn(g["a_full"][rows], r["a_full"], "config1 dual full")
+    assert_close_attn(g["a_loc"][rows], r["a_loc"], "config1 dual loc")
+    assert np.isfinite(g["disc"]).all()
