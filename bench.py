@@ -1,0 +1,440 @@
+"""Chunk-step benchmark of the ISPA hot path on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--model 1.3b|14b]
+
+One step = one pass of the whole hot path over one chunk of a 1.3B-shaped
+layer stack (12 heads x 128, 1560 tokens/frame, 3-frame chunk = 4680 queries):
+  * F-layer attention over an 18-frame ring (28080 + 4680 keys),
+  * L-layer attention over its 6-frame window ring (9360 + 4680 keys),
+  * warmup dual attention on an 18-frame ring (local = chunk + 6 frames, hist = 12 frames),
+  * least-squares accumulation of that layer's (A_loc, A_full) over its 4680 tokens,
+  * KV append of the finished chunk into all three rings (one launch).
+The rings stay in steady state (each append evicts the oldest 3 frames).
+value = attention FLOPs of the three modes (4*Nq*Nk*d*H each) / device time of the step.
+L2 is flushed (256 MB write) between timed steps, outside the timed events.
+Inputs are synthetic (seeded N(0,1) q/k/v with per-frame key offsets), bf16.
+
+Under torchrun (N > 1) every rank runs an independent replica on its own GPU
+(the path has no exchange step); timing is max over ranks and value sums ranks.
+--impl reference times the fp64 CPU oracle on a bounded sample of the same step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "chunk-step attention TFLOP/s (full/local/dual) and % of GB300 dense bf16 peak"
+UNIT = "TFLOP/s"
+
+MODELS = {
+    # name: (heads, head_dim, tokens/frame, chunk frames, F-ring frames, window frames)
+    "1.3b": (12, 128, 1560, 3, 18, 6),
+    "14b": (40, 128, 1560, 3, 18, 6),
+}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(bf16=d["bf16_tflops"], bf16_sustained=d.get("bf16_tflops_sustained"), hbm=d["hbm_gbs"],
+                    source="measured")
+    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+
+
+def attn_flops(nq, nk, d, H):
+    return 4.0 * nq * nk * d * H
+
+
+def workload(model):
+    H, d, P, L, F, Wn = MODELS[model]
+    nq = L * P
+    return dict(H=H, d=d, P=P, L=L, F=F, W=Wn, nq=nq, D=H * d,
+                nk_full=F * P + nq, nk_local=Wn * P + nq,
+                flops_full=attn_flops(nq, F * P + nq, d, H),
+                flops_local=attn_flops(nq, Wn * P + nq, d, H),
+                flops_dual=attn_flops(nq, F * P + nq, d, H))
+
+
+# ---------------------------------------------------------------- clocks sampler
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines: list[str] = []
+        self.t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.idx), "-lms", "200"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.t:
+            self.t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return dict(sm_mhz=statistics.median(sm), sm_max_mhz=max(mx), reasons=sorted(reasons), samples=len(sm))
+
+
+def physical_gpu_index(local_rank: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        parts = [p for p in vis.split(",") if p.strip()]
+        if local_rank < len(parts) and parts[local_rank].strip().isdigit():
+            return int(parts[local_rank])
+    return local_rank
+
+
+# ---------------------------------------------------------------- our arm
+class StepRunner:
+    """Device buffers and the libispa call sequence of one chunk step."""
+
+    def __init__(self, wl, device, seed=0):
+        import torch
+
+        from paper_2607_00712_gb300 import abi, synth
+        from paper_2607_00712_gb300.device import LS, Ring, Window, bf16_tensor
+        self.abi, self.torch = abi, torch
+        H, d, P, L, F, Wn, nq, D = (wl[k] for k in ("H", "d", "P", "L", "F", "W", "nq", "D"))
+        self.wl = wl
+        self.win = Window(0, Wn)
+        # three layers: F-layer (18-frame ring), L-layer (window ring), warmup layer (18-frame ring)
+        self.rings = [Ring(H, d, P, F, 0, device), Ring(H, d, P, Wn, 0, device), Ring(H, d, P, F, 0, device)]
+        self.inputs = []
+        self.debug = False
+        for li, ring in enumerate(self.rings):
+            t0 = time.perf_counter()
+            s = synth.make_step(seed * 100 + li, ring.c.capacity_frames, P, H, d, L)
+            log(f"[bench] inputs of layer {li} drawn in {time.perf_counter() - t0:.1f} s")
+            for f0 in range(0, ring.c.capacity_frames, L):
+                n = min(L, ring.c.capacity_frames - f0)
+                abi.ispa_kv_append(ring.c, bf16_tensor(s.k_hist[f0 * P:(f0 + n) * P], device),
+                                   bf16_tensor(s.v_hist[f0 * P:(f0 + n) * P], device), n)
+            self.inputs.append((bf16_tensor(s.q, device), bf16_tensor(s.k_cur, device), bf16_tensor(s.v_cur, device)))
+        bf = torch.bfloat16
+        self.out_full = torch.empty(nq, D, dtype=bf, device=device)
+        self.out_local = torch.empty(nq, D, dtype=bf, device=device)
+        self.a_full = torch.empty(nq, D, dtype=bf, device=device)
+        self.a_loc = torch.empty(nq, D, dtype=bf, device=device)
+        self.disc = torch.empty(nq, dtype=torch.float32, device=device)
+        self.disc_sum = torch.zeros(1, dtype=torch.float32, device=device)
+        self.dual_wsb = abi.ispa_attn_dual_workspace_size(H, nq)
+        self.dual_ws = torch.empty(self.dual_wsb, dtype=torch.uint8, device=device)
+        self.ls = LS(D, device)
+        self.ls_wsb = abi.ispa_ls_accumulate_workspace_size(D, nq)
+        self.ls_ws = torch.empty(self.ls_wsb, dtype=torch.uint8, device=device)
+        self.ring_arr = (abi.KVRing * 3)()
+        self.stream = torch.cuda.current_stream(device)
+        self.launches_per_step = 7   # 3 attention + disc reduce + split + gram + append
+        torch.cuda.synchronize(device)
+
+    def step(self, ev=None):
+        """Enqueue one step; ev = list of 6 events to record between the calls (or None)."""
+        abi, nq = self.abi, self.wl["nq"]
+        s = self.stream
+        if self.debug:
+            def rec(i):
+                self.torch.cuda.synchronize()
+                st, code = abi.ispa_last_device_error()
+                log(f"[bench]   call {i} done, device status {st}/{code}")
+        else:
+            rec = (lambda i: ev[i].record(s)) if ev else (lambda i: None)
+        rec(0)
+        q, kc, vc = self.inputs[0]
+        abi.ispa_attn_full(self.rings[0].c, q, kc, vc, nq, 0.0, self.out_full, None, s)
+        rec(1)
+        q, kc, vc = self.inputs[1]
+        abi.ispa_attn_local(self.rings[1].c, self.win, q, kc, vc, nq, 0.0, self.out_local, None, s)
+        rec(2)
+        q, kc, vc = self.inputs[2]
+        abi.ispa_attn_dual(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, self.a_full, self.a_loc, self.disc,
+                           self.disc_sum, None, None, self.dual_ws, self.dual_wsb, s)
+        rec(3)
+        abi.ispa_ls_accumulate(self.ls.c, self.a_loc, self.a_full, nq, self.ls_ws, self.ls_wsb, s)
+        rec(4)
+        for i in range(3):
+            self.ring_arr[i] = self.rings[i].c
+        abi.ispa_kv_append_layers(self.ring_arr, [x[1] for x in self.inputs], [x[2] for x in self.inputs],
+                                  self.wl["L"], s)
+        for i in range(3):
+            self.rings[i].c.frames_written = self.ring_arr[i].frames_written
+        rec(5)
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    from paper_2607_00712_gb300 import abi
+    from paper_2607_00712_gb300.build import build_library
+    t_start = time.perf_counter()
+    build_library()
+    abi.lib()
+    wl = workload(args.model)
+    pk = peaks()
+    r = StepRunner(wl, device)
+    log(f"[bench] set-up done in {time.perf_counter() - t_start:.1f} s")
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=device)
+
+    for i in range(args.warmup):
+        r.debug = i == 0
+        r.step()
+        r.debug = False
+        torch.cuda.synchronize(device)
+        log(f"[bench] warmup step {i} done at {time.perf_counter() - t_start:.1f} s")
+    st, code = abi.ispa_last_device_error()
+    if st != abi.ISPA_OK:
+        raise RuntimeError(f"device error after warmup: {code}")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    sampler = ClockSampler(physical_gpu_index(local_rank)) if rank == 0 else None
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(device)
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.fill_(float(k))          # L2 flush, outside the step's events
+        r.step(evs[k])
+    torch.cuda.synchronize(device)
+    wall = time.perf_counter() - t0
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop() if sampler else None
+    st, code = abi.ispa_last_device_error()
+    if st != abi.ISPA_OK:
+        raise RuntimeError(f"device error in timed region: {code}")
+
+    seg = np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(5)] for k in range(args.steps)])
+    step_ms = seg.sum(axis=1)
+    total_ms = float(step_ms.sum())
+    if world > 1:
+        t = torch.tensor([total_ms], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    flops_step = wl["flops_full"] + wl["flops_local"] + wl["flops_dual"]
+    ms_per_step = total_ms / args.steps
+    value = world * flops_step / (ms_per_step * 1e-3) / 1e12
+    mean = seg.mean(axis=0)
+    modes = dict(
+        full=dict(ms=mean[0], tflops=wl["flops_full"] / (mean[0] * 1e-3) / 1e12, nk=wl["nk_full"]),
+        local=dict(ms=mean[1], tflops=wl["flops_local"] / (mean[1] * 1e-3) / 1e12, nk=wl["nk_local"]),
+        dual=dict(ms=mean[2], tflops=wl["flops_dual"] / (mean[2] * 1e-3) / 1e12, nk=wl["nk_full"]),
+        ls_accumulate=dict(ms=mean[3]),
+        kv_append=dict(ms=mean[4], gbs=3 * 2 * 2 * wl["nq"] * wl["D"] * 2 / (mean[4] * 1e-3) / 1e9),
+    )
+    for m in modes.values():
+        for k_, v_ in list(m.items()):
+            if isinstance(v_, float):
+                m[k_] = round(v_, 4)
+    achieved = modes["full"]["tflops"]
+    roofline = dict(bound="tensor", achieved=round(achieved, 2), peak=pk["bf16"], unit="TFLOP/s",
+                    frac=round(achieved / pk["bf16"], 4), traffic=None,
+                    kernel="attn_kernel<128> (F-layer launch)", peak_source=pk["source"] + " burst bf16",
+                    frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
+
+    log(f"[bench] timed steps done at {time.perf_counter() - t_start:.1f} s")
+    e2e = run_e2e(r, args, device, flops_step, world)
+    log(f"[bench] e2e done at {time.perf_counter() - t_start:.1f} s")
+
+    result = dict(metric=METRIC, value=round(value, 3), unit=UNIT, n_gpus=world, steps=args.steps,
+                  warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
+                  scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
+                  config=dict(workload=f"ISPA chunk step, {args.model}-shaped layer stack (F + L + dual + LS + append)",
+                              heads=wl["H"], head_dim=wl["d"], tokens_per_frame=wl["P"], n_q=wl["nq"],
+                              f_ring_frames=wl["F"], window_frames=wl["W"], parallelism=f"replicas x{world}",
+                              l2="flushed between steps (256 MB write outside timed events)"),
+                  modes=modes, roofline=roofline, e2e=e2e,
+                  gpu_launches=r.launches_per_step * args.steps, clocks=clocks,
+                  wall_s=round(wall, 3))
+    if rank == 0:
+        if args.cpu_baseline:
+            result["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_rows)
+        print(json.dumps(result), flush=True)
+
+
+def run_e2e(r, args, device, flops_step, world):
+    """The same step through the C-ABI with pinned host inputs / outputs copied inside the timed region."""
+    import torch
+    host_in = [[t.cpu().pin_memory() for t in trip] for trip in r.inputs]
+    outs = [r.out_full, r.out_local, r.a_full, r.a_loc, r.disc]
+    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs]
+    h2d = sum(t.numel() * t.element_size() for trip in host_in for t in trip)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    s = r.stream
+    n = max(3, min(args.steps, 20))
+
+    def one():
+        for trip_h, trip_d in zip(host_in, r.inputs):
+            for h, dv in zip(trip_h, trip_d):
+                dv.copy_(h, non_blocking=True)
+        r.step()
+        for h, dv in zip(host_out, outs):
+            h.copy_(dv, non_blocking=True)
+    one()
+    torch.cuda.synchronize(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(s)
+    for _ in range(n):
+        one()
+    e1.record(s)
+    torch.cuda.synchronize(device)
+    ms = e0.elapsed_time(e1) / n
+    return dict(value=round(world * flops_step / (ms * 1e-3) / 1e12, 3), unit=UNIT, h2d_bytes_per_step=h2d,
+                d2h_bytes_per_step=d2h, ms_per_step=round(ms, 4), steps=n)
+
+
+# ---------------------------------------------------------------- oracle legs
+def _oracle_sample(wl, rows_per_mode, seed=0):
+    """Inputs of one bounded oracle sample: the three layers' steps, sampled query rows."""
+    from paper_2607_00712_gb300 import synth
+    H, d, P, L, F, Wn = (wl[k] for k in ("H", "d", "P", "L", "F", "W"))
+    steps = [synth.make_step(seed * 100 + li, cap, P, H, d, L) for li, cap in enumerate([F, Wn, F])]
+    rng = np.random.default_rng(seed)
+    rows = np.sort(rng.choice(wl["nq"], rows_per_mode, replace=False))
+    return steps, rows
+
+
+def _oracle_step(wl, steps, rows):
+    from oracle import attention as oat
+    from oracle import ls as ols
+    P, Wn = wl["P"], wl["W"]
+    s0, s1, s2 = steps
+    oat.attn_full(s0.q, s0.k_hist, s0.v_hist, s0.k_cur, s0.v_cur, P, rows=rows)
+    oat.attn_local(s1.q, s1.k_hist, s1.v_hist, s1.k_cur, s1.v_cur, P, 0, Wn, rows=rows)
+    r = oat.attn_dual(s2.q, s2.k_hist, s2.v_hist, s2.k_cur, s2.v_cur, P, 0, Wn, rows=rows)
+    n = len(rows)
+    st = ols.ls_state(wl["D"])
+    ols.ls_accumulate(st, r["a_loc"].reshape(n, -1), r["a_full"].reshape(n, -1))
+    # algorithmic attention FLOPs of the sampled rows (same count as the GPU metric)
+    return (wl["flops_full"] + wl["flops_local"] + wl["flops_dual"]) * n / wl["nq"]
+
+
+def cpu_baseline(wl, rows):
+    steps, rs = _oracle_sample(wl, rows)
+    t0 = time.perf_counter()
+    flops = _oracle_step(wl, steps, rs)
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return dict(value=round(flops / dt / 1e12, 6), unit=UNIT, cores=cores, kind="oracle",
+                sample=f"{rows} of {wl['nq']} query rows of each mode (full, local, dual) x all heads, "
+                       f"plus LS accumulation of those rows; fp64 numpy, {dt:.1f} s",
+                seconds=round(dt, 2))
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    wl = workload(args.model)
+    rows = args.ref_rows
+    steps, rs = _oracle_sample(wl, rows)
+    for _ in range(args.warmup if args.warmup < 1 else 1):
+        _oracle_step(wl, steps, rs[:8])
+    t0 = time.perf_counter()
+    flops = 0.0
+    for _ in range(args.steps):
+        flops += _oracle_step(wl, steps, rs)
+    dt = time.perf_counter() - t0
+    value = flops / dt / 1e12
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    res = dict(impl="reference", metric=METRIC, value=round(value, 6), unit=UNIT, n_gpus=world, steps=args.steps,
+               warmup=args.warmup, ms_per_step=round(dt / args.steps * 1e3, 2), higher_is_better=True,
+               scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+               config=dict(workload=f"ISPA chunk step, {args.model}-shaped layer stack (F + L + dual + LS)",
+                           heads=wl["H"], head_dim=wl["d"], tokens_per_frame=wl["P"], n_q=wl["nq"],
+                           sample_rows=rows),
+               cpu_baseline=dict(value=round(value, 6), unit=UNIT, cores=cores, kind="oracle",
+                                 sample=f"{rows} query rows per mode per step"),
+               e2e=dict(value=round(value, 6), unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+    print(json.dumps(res), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--model", choices=sorted(MODELS), default="1.3b")
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--cpu-sample-rows", type=int, default=128)
+    ap.add_argument("--ref-rows", type=int, default=32)
+    ap.add_argument("--watchdog", type=float, default=300.0, help="dump Python stacks after this many s")
+    args = ap.parse_args()
+    import faulthandler
+    faulthandler.dump_traceback_later(args.watchdog, exit=False)
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

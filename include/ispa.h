@@ -147,6 +147,19 @@ ISPA_API uint64_t ispa_set_wait_limit_ns(uint64_t ns);
  * and status path without touching any other state. */
 ISPA_API ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream);
 
+/* Copy (without clearing) the device error record of the current device:
+ * rec8[0] = code (0 none, 1 timeout), then the first failing wait: [1] wait
+ * site, [2] blockIdx.x, [3] blockIdx.y, [4] threadIdx.x, [5] barrier shared
+ * address, [6] parity, [7] tile index.  rec8: host array of 8 int32.
+ * Synchronises like ispa_last_device_error. */
+ISPA_API ispa_status ispa_debug_error_record(int32_t* rec8);
+
+/* Debug aid: counters (a device-accessible pointer to host-mapped memory,
+ * n_slots * 4 uint32) that the tcgen05 kernels bump per CTA: [0] started,
+ * [1] TMEM allocated, [2] finished.  Each launch takes the next slot in turn.
+ * NULL / 0 turns it off (the default). */
+ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots);
+
 /* Bytes of one ring's K and V buffers together (2 * H * cap * P * d * 2). */
 ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);
 

@@ -69,6 +69,8 @@ _SIGS = {
     "ispa_last_device_error": (c_int32, [POINTER(c_int32)]),
     "ispa_set_wait_limit_ns": (c_uint64, [c_uint64]),
     "ispa_debug_wait_probe": (c_int32, [c_uint64, c_void_p]),
+    "ispa_debug_error_record": (c_int32, [POINTER(c_int32)]),
+    "ispa_debug_set_heartbeat": (c_int32, [c_void_p, c_int32]),
     "ispa_ring_bytes": (c_size_t, [POINTER(KVRing)]),
     "ispa_ring_slot": (c_int32, [POINTER(KVRing), c_int64]),
     "ispa_window_resolve": (c_int32, [POINTER(KVRing), Window, POINTER(KeySets)]),
@@ -148,6 +150,16 @@ def ispa_set_wait_limit_ns(ns: int) -> int:
 
 def ispa_debug_wait_probe(limit_ns: int, stream=None) -> None:
     _check(lib().ispa_debug_wait_probe(limit_ns, _stream(stream)), "ispa_debug_wait_probe")
+
+
+def ispa_debug_error_record() -> list[int]:
+    rec = (c_int32 * 8)()
+    _check(lib().ispa_debug_error_record(rec), "ispa_debug_error_record")
+    return list(rec)
+
+
+def ispa_debug_set_heartbeat(counters, n_slots: int) -> None:
+    _check(lib().ispa_debug_set_heartbeat(_ptr(counters), n_slots), "ispa_debug_set_heartbeat")
 
 
 def ispa_ring_bytes(ring: KVRing) -> int:

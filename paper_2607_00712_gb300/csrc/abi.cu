@@ -15,7 +15,7 @@
 
 namespace ispa {
 
-static __device__ int g_status;  // device error word (DEVERR_*), one per device
+static __device__ int g_status[8];  // device error record (DEVERR_* + location), one per device
 
 namespace {
 
@@ -46,6 +46,20 @@ EncodeTiledFn encode_fn() {
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_limit; }
+
+namespace {
+uint32_t* g_hb = nullptr;   // host-mapped heartbeat buffer (device address), debug only
+int g_hb_slots = 0;
+int g_hb_next = 0;
+}  // namespace
+
+uint32_t* next_heartbeat_slot(uint32_t kernel_tag) {
+  if (!g_hb || g_hb_slots <= 0) return nullptr;
+  uint32_t* slot = g_hb + 4 * (g_hb_next % g_hb_slots);
+  ++g_hb_next;
+  (void)kernel_tag;
+  return slot;
+}
 
 int* device_status_ptr() {
   static int* ptrs[64] = {};
@@ -222,6 +236,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   p.disc_part = disc_part;
   p.status = device_status_ptr();
   if (!p.status) return ISPA_ERR_CUDA;
+  p.heartbeat = next_heartbeat_slot(1);
 
   const uint64_t row_b = static_cast<uint64_t>(HD) * 2;
   const uint64_t ring_tok = static_cast<uint64_t>(ring->capacity_frames) * P;
@@ -273,12 +288,26 @@ const char* ispa_status_string(ispa_status s) {
 }
 
 ispa_status ispa_last_device_error(int32_t* code) {
-  int v = 0;
-  if (cudaMemcpyFromSymbol(&v, g_status, sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
-  const int zero = 0;
-  if (cudaMemcpyToSymbol(g_status, &zero, sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
-  if (code) *code = v;
-  if (v == DEVERR_TIMEOUT) return ISPA_ERR_TIMEOUT;
+  int rec[8] = {};
+  if (cudaMemcpyFromSymbol(rec, g_status, sizeof(rec)) != cudaSuccess) return ISPA_ERR_CUDA;
+  const int zero[8] = {};
+  if (cudaMemcpyToSymbol(g_status, zero, sizeof(zero)) != cudaSuccess) return ISPA_ERR_CUDA;
+  if (code) *code = rec[0];
+  if (rec[0] == DEVERR_TIMEOUT) return ISPA_ERR_TIMEOUT;
+  return ISPA_OK;
+}
+
+ispa_status ispa_debug_error_record(int32_t* rec8) {
+  if (!rec8) return ISPA_ERR_INVALID_ARG;
+  if (cudaMemcpyFromSymbol(rec8, g_status, 8 * sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots) {
+  if ((counters == nullptr) != (n_slots <= 0)) return ISPA_ERR_INVALID_ARG;
+  g_hb = counters;
+  g_hb_slots = n_slots;
+  g_hb_next = 0;
   return ISPA_OK;
 }
 
@@ -427,7 +456,7 @@ ispa_status ispa_ls_accumulate(ispa_ls_state* st, const void* a_loc, const void*
   int* status = device_status_ptr();
   if (!status) return ISPA_ERR_CUDA;
   if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, st->gram, status, g_wait_limit,
-                           stream) != cudaSuccess)
+                           next_heartbeat_slot(2), stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   st->n_tokens += T;
   return ISPA_OK;

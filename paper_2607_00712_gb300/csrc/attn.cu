@@ -142,9 +142,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if (threadIdx.x == 0) heartbeat(p.heartbeat, 0);
   if (warp == WARP_MMA) {
     tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
     tmem_relinquish();
+    if (lane == 0) heartbeat(p.heartbeat, 1);
   }
   if (warp == WARP_TMA && lane == 0) {
     tma_prefetch_desc(&tm_q);
@@ -173,7 +175,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const bool chunk = p.seg[seg].src != 0;
         const int row = p.seg[seg].start + off;
         const int ks = j % C::KST, vs = j % C::VST;
-        if (!mbar_wait(b.k_empty0 + 8 * ks, ((j / C::KST) & 1) ^ 1, wc)) break;
+        if (!mbar_wait(b.k_empty0 + 8 * ks, ((j / C::KST) & 1) ^ 1, wc, 1, j)) break;
         mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::TILE);
         const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
 #pragma unroll
@@ -182,7 +184,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           else tma_load_3d(sK + x * C::BOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
         }
         nk = j + 1;
-        if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc)) break;
+        if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
         mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::TILE);
         const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
 #pragma unroll
@@ -206,11 +208,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // ------------------------------------------------------------ UMMA issuer
     if (lane == 0) {
       const uint32_t sQ = sbase + C::OFF_Q;
-      bool ok = mbar_wait(b.q_full, 0, wc);
+      bool ok = mbar_wait(b.q_full, 0, wc, 3, 0);
       tc_fence_after();
       auto issue_s = [&](int j) -> bool {
         const int ks = j % C::KST;
-        if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc)) return false;
+        if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc, 4, j)) return false;
         tc_fence_after();
         const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
         const uint32_t d = tmem + C::COL_S0 + (j & 1) * 128;
@@ -228,8 +230,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       if (ok && n_tiles > 1) ok = issue_s(1);
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int vs = j % C::VST;
-        if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc)) break;
-        if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc)) break;
+        if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
+        if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
         tc_fence_after();
         const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
         const uint32_t a = tmem + C::COL_P0 + (j & 1) * 64;
@@ -306,12 +308,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int sb = j & 1;
       if (p.dual && j == p.n_local_tiles && j > 0) {
         // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc));
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 7, j));
         if (!ok) break;
         tc_fence_after();
         emit(p.out_loc, p.lse_loc, false);
       }
-      ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc));
+      ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
       if (!ok) break;
       tc_fence_after();
       const int valid = min(BN, p.seg[seg].count - off);
@@ -340,12 +342,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
       if (j == 0) {
         m_run = m_tile;
-      } else if (m_tile > m_run + RESCALE_THRESHOLD) {
-        // Lazy rescale: O holds PV of tiles 0..j-1 once PV_{j-1} has completed.
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc));
+      } else if (__any_sync(0xffffffffu, m_tile > m_run + RESCALE_THRESHOLD)) {
+        // Lazy rescale, decided per warp (the TMEM accesses are warp-collective):
+        // O holds PV of tiles 0..j-1 once PV_{j-1} has completed.  Lanes whose max
+        // did not grow keep alpha = 1.
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 9, j));
         if (!ok) break;
         tc_fence_after();
-        const float alpha = ex2_approx(m_run - m_tile);
+        const float m_new = fmaxf(m_run, m_tile);
+        const float alpha = ex2_approx(m_run - m_new);
         l_run *= alpha;
 #pragma unroll 1
         for (int c = 0; c < HD / 32; ++c) {
@@ -357,11 +362,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           tmem_st32(trow + C::COL_O + 32 * c, r);
         }
         tmem_wait_st();
-        m_run = m_tile;
+        m_run = m_new;
       }
       // P_j goes to TMEM buffer sb, last read by PV_{j-2}.
       if (j >= 2) {
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc));
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc, 10, j));
         if (!ok) break;
         tc_fence_after();
       }
@@ -388,7 +393,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
     if (ok) {
       const int jl = n_tiles - 1;
-      ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc));
+      ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc, 11, jl));
       if (ok) {
         tc_fence_after();
         if (p.dual && p.n_local_tiles >= n_tiles) emit(p.out_loc, p.lse_loc, false);
@@ -402,6 +407,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   if (warp == WARP_MMA) {
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
+    if (lane == 0) heartbeat(p.heartbeat, 2);
   }
 }
 

@@ -61,6 +61,7 @@ struct GramParams {
   float* gram;        // [2D][2D]
   int* status;
   uint64_t wait_limit_ns;
+  uint32_t* heartbeat;
 };
 
 // Decode blockIdx.x into (kind, row block, col block).  Items: upper G tiles,
@@ -158,9 +159,11 @@ __global__ void __launch_bounds__(G_THREADS, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if (threadIdx.x == 0) heartbeat(p.heartbeat, 0);
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
     tmem_relinquish();
+    if (lane == 0) heartbeat(p.heartbeat, 1);
   }
   tc_fence_before();
   __syncthreads();
@@ -176,7 +179,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
         const int pass = s / n_kt;
         const int tok = (kt0 + s % n_kt) * GK;
         const int st = s % GST;
-        if (!mbar_wait(empty0 + 8 * st, ((s / GST) & 1) ^ 1, wc)) break;
+        if (!mbar_wait(empty0 + 8 * st, ((s / GST) & 1) ^ 1, wc, 21, s)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
         const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
         const CUtensorMap* ma = maps[kPasses[kind][pass].a];
@@ -196,7 +199,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
       bool ok = true;
       for (int s = 0; s < total_steps; ++s) {
         const int st = s % GST;
-        if (!mbar_wait(full0 + 8 * st, (s / GST) & 1, wc)) {
+        if (!mbar_wait(full0 + 8 * st, (s / GST) & 1, wc, 22, s)) {
           ok = false;
           break;
         }
@@ -217,7 +220,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
     // epilogue: warp w reads TMEM lanes 32*(w%4) .. +31 = output rows
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, wc));
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, wc, 23, 0));
     if (ok) {
       tc_fence_after();
       const int D = p.D;
@@ -244,6 +247,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
+    if (lane == 0) heartbeat(p.heartbeat, 2);
   }
 }
 
@@ -255,7 +259,7 @@ size_t ls_accumulate_ws_bytes(int32_t D, int64_t T) {
 
 template <int BN>
 static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
-                               float* gram, int* status, uint64_t wait_limit_ns, cudaStream_t s) {
+                               float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
   using C = GCfg<BN>;
   static bool attr_done[64] = {};
   int dev = 0, sms = 152;
@@ -287,13 +291,15 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   p.gram = gram;
   p.status = status;
   p.wait_limit_ns = wait_limit_ns;
+  p.heartbeat = hb;
   dim3 grid(n_items, splits);
   gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(ta, th, tl, p);
   return cudaGetLastError();
 }
 
 cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full, void* ws,
-                                 float* gram, int* status, uint64_t wait_limit_ns, cudaStream_t s) {
+                                 float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
+                                 cudaStream_t s) {
   const size_t one = ls_accumulate_ws_bytes(D, T) / 2;
   uint8_t* hi = static_cast<uint8_t*>(ws);
   uint8_t* lo = hi + one;
@@ -308,8 +314,8 @@ cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const 
       reinterpret_cast<uint4*>(lo), n_words);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (D % 256 == 0) return launch_gram<256>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, s);
-  return launch_gram<128>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, s);
+  if (D % 256 == 0) return launch_gram<256>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
+  return launch_gram<128>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
 }
 
 }  // namespace ispa

@@ -39,7 +39,8 @@ struct AttnParams {
   float* lse;              // [H][n_q] or null
   float* lse_loc;          // [H][n_q] or null (dual)
   float* disc_part;        // [H][n_q] per-head sum of squared discrepancy (dual)
-  int* status;             // library status word
+  int* status;             // library status record
+  uint32_t* heartbeat;     // debug counters (host-mapped) or null
 };
 
 // Launch the attention kernel.  tensor maps are encoded by the caller.
@@ -74,7 +75,7 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 // Accumulate the upper blocks of [A | dlt]^T [A | dlt] into the fp32 state.
 cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full,
                                  void* ws, float* gram, int* status, uint64_t wait_limit_ns,
-                                 cudaStream_t s);
+                                 uint32_t* heartbeat, cudaStream_t s);
 size_t ls_accumulate_ws_bytes(int32_t D, int64_t T);
 
 size_t ls_solve_ws_bytes(int32_t D, int32_t d_out);
@@ -90,5 +91,6 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, 
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();
+uint32_t* next_heartbeat_slot(uint32_t kernel_tag);  // null unless a heartbeat buffer is set
 
 }  // namespace ispa

@@ -55,9 +55,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // Context of the bounded waits of one CTA.
 struct WaitCtx {
   volatile int* abort;     // shared-memory abort flag of the CTA
-  int* status;             // library status word (global)
+  int* status;             // library status record (global): see record_error
   uint64_t limit_ns;       // give up after this long
 };
+
+// status[0] = code; the first CTA to fail also records where:
+// status[1] = wait site, [2] = blockIdx.x, [3] = blockIdx.y, [4] = threadIdx.x,
+// [5] = barrier smem address, [6] = parity, [7] = kernel-defined detail (tile).
+__device__ __forceinline__ void record_error(int* status, int code, int site, uint32_t bar, uint32_t parity,
+                                             int detail) {
+  if (atomicCAS(status, DEVERR_NONE, code) == DEVERR_NONE) {
+    status[1] = site;
+    status[2] = static_cast<int>(blockIdx.x);
+    status[3] = static_cast<int>(blockIdx.y);
+    status[4] = static_cast<int>(threadIdx.x);
+    status[5] = static_cast<int>(bar);
+    status[6] = static_cast<int>(parity);
+    status[7] = detail;
+    __threadfence();
+  }
+}
 
 __device__ __forceinline__ void raise_abort(const WaitCtx& w, int code) {
   *w.abort = 1;
@@ -66,8 +83,10 @@ __device__ __forceinline__ void raise_abort(const WaitCtx& w, int code) {
 
 // Wait for the phase of `bar` with the given parity to complete.  Returns
 // false (and raises the abort flag) once the limit has passed, or as soon as
-// another role of the CTA has aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& w) {
+// another role of the CTA has aborted.  `site` and `detail` identify the wait
+// in the error record.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& w, int site = 0,
+                                          int detail = 0) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
@@ -75,10 +94,20 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const W
     if ((i & 63) == 0) {
       if (*w.abort) return false;
       if (globaltimer_ns() - t0 > w.limit_ns) {
-        raise_abort(w, DEVERR_TIMEOUT);
+        *w.abort = 1;
+        record_error(w.status, DEVERR_TIMEOUT, site, bar, parity, detail);
         return false;
       }
     }
+  }
+}
+
+// Heartbeat counters in host-visible memory (debug aid): hb[0] += 1 at CTA
+// start, hb[1] after the TMEM allocation, hb[2] at CTA exit.
+__device__ __forceinline__ void heartbeat(uint32_t* hb, int idx) {
+  if (hb) {
+    atomicAdd_system(hb + idx, 1u);
+    __threadfence_system();
   }
 }
 

@@ -6,7 +6,10 @@ Both the CUDA path and the fp64 oracle consume exactly the arrays made here.
 
 Input recipe (stand-in for the post-RoPE activations of an autoregressive
 video DiT, Sec. 2 "KV injection", Eq. 3):
-  * q, k, v ~ N(0, 1), drawn in fp32 from numpy's PCG64 with the given seed;
+  * q, k, v ~ N(0, 1), drawn in fp32 with numpy's PCG64: each array gets its
+    own child of SeedSequence(seed), split into 2^20-value chunks with one
+    grandchild stream each (drawn in parallel threads, so the values depend
+    only on the seed and the array shapes);
   * every key of frame f and head h additionally gets an offset vector
     mu[f, h, :] ~ N(0, 0.5^2) (0.5 read as the standard deviation), so the
     softmax over frames is non-uniform;
@@ -16,9 +19,13 @@ Token-major layout everywhere: a block of n frames is [n*P, H, d].
 """
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass
 
 import numpy as np
+
+_CHUNK = 1 << 20
 
 KEY_OFFSET_STD = 0.5
 
@@ -26,9 +33,13 @@ KEY_OFFSET_STD = 0.5
 def bf16_round(x: np.ndarray) -> np.ndarray:
     """Round fp32 values to the nearest bfloat16 (ties to even); returns fp32."""
     x = np.ascontiguousarray(x, dtype=np.float32)
-    u = x.view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
-    return u.astype(np.uint32).view(np.float32).reshape(x.shape)
+    u = x.view(np.uint32)
+    # finite inputs: the sum stays below 2^32 (only NaN bit patterns are above 0xFFFF0000)
+    r = (u >> 16) & np.uint32(1)
+    r += np.uint32(0x7FFF)
+    r += u
+    r &= np.uint32(0xFFFF0000)
+    return r.view(np.float32).reshape(x.shape)
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -42,19 +53,36 @@ def bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (np.ascontiguousarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
 
 
-def _normal(rng: np.random.Generator, shape, std: float = 1.0) -> np.ndarray:
-    a = rng.standard_normal(size=shape, dtype=np.float32)
+def _normal(ss: np.random.SeedSequence, shape, std: float = 1.0) -> np.ndarray:
+    """N(0, std^2) fp32 array of the given shape from the seed sequence ss."""
+    n = int(np.prod(shape))
+    out = np.empty(n, np.float32)
+    n_chunks = max(1, (n + _CHUNK - 1) // _CHUNK)
+    kids = ss.spawn(n_chunks)
+
+    def work(i):
+        g = np.random.Generator(np.random.PCG64(kids[i]))
+        lo, hi = i * _CHUNK, min(n, (i + 1) * _CHUNK)
+        if hi > lo:
+            g.standard_normal(out=out[lo:hi], dtype=np.float32)
+
+    if n_chunks == 1:
+        work(0)
+    else:
+        with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+            list(ex.map(work, range(n_chunks)))
     if std != 1.0:
-        a *= np.float32(std)
-    return a
+        out *= np.float32(std)
+    return out.reshape(shape)
 
 
-def frame_block(rng: np.random.Generator, n_frames: int, P: int, H: int, d: int,
+def frame_block(ss: np.random.SeedSequence, n_frames: int, P: int, H: int, d: int,
                 with_offset: bool = True) -> np.ndarray:
     """Keys of n_frames frames, [n*P, H, d] fp32, with the per-(frame, head) offset."""
-    k = _normal(rng, (n_frames, P, H, d))
+    a, b = ss.spawn(2)
+    k = _normal(a, (n_frames, P, H, d))
     if with_offset:
-        mu = _normal(rng, (n_frames, 1, H, d), KEY_OFFSET_STD)
+        mu = _normal(b, (n_frames, 1, H, d), KEY_OFFSET_STD)
         k += mu
     return k.reshape(n_frames * P, H, d)
 
@@ -87,13 +115,13 @@ class StepInputs:
 def make_step(seed: int, n_past_frames: int, P: int, H: int, d: int,
               n_chunk_frames: int = 3) -> StepInputs:
     """Seeded inputs of one chunk step (recipe in the module docstring)."""
-    rng = np.random.Generator(np.random.PCG64(seed))
+    s_q, s_kc, s_vc, s_kh, s_vh = np.random.SeedSequence(seed).spawn(5)
     nq = n_chunk_frames * P
-    q = bf16_round(_normal(rng, (nq, H, d)))
-    k_cur = bf16_round(frame_block(rng, n_chunk_frames, P, H, d))
-    v_cur = bf16_round(_normal(rng, (nq, H, d)))
-    k_hist = bf16_round(frame_block(rng, n_past_frames, P, H, d))
-    v_hist = bf16_round(_normal(rng, (n_past_frames * P, H, d)))
+    q = bf16_round(_normal(s_q, (nq, H, d)))
+    k_cur = bf16_round(frame_block(s_kc, n_chunk_frames, P, H, d))
+    v_cur = bf16_round(_normal(s_vc, (nq, H, d)))
+    k_hist = bf16_round(frame_block(s_kh, n_past_frames, P, H, d))
+    v_hist = bf16_round(_normal(s_vh, (n_past_frames * P, H, d)))
     return StepInputs(q, k_cur, v_cur, k_hist, v_hist, P, H, d)
 
 
@@ -103,13 +131,12 @@ def make_activations(seed: int, T: int, D: int, coupling: float = 0.5):
     A_full = A_loc + coupling * N(0,1) noise, so the discrepancy is of the size
     an attention output sees when half its history is removed.
     """
-    rng = np.random.Generator(np.random.PCG64(seed))
-    a_loc = bf16_round(_normal(rng, (T, D)))
-    a_full = bf16_round(a_loc + _normal(rng, (T, D), coupling))
+    s_a, s_n = np.random.SeedSequence(seed).spawn(2)
+    a_loc = bf16_round(_normal(s_a, (T, D)))
+    a_full = bf16_round(a_loc + _normal(s_n, (T, D), coupling))
     return a_loc, a_full
 
 
 def make_weight(seed: int, D: int, D_out: int) -> np.ndarray:
     """A synthetic output-projection weight W [D, D_out] (row-vector convention A @ W)."""
-    rng = np.random.Generator(np.random.PCG64(seed))
-    return (_normal(rng, (D, D_out)) / np.float32(np.sqrt(D))).astype(np.float32)
+    return (_normal(np.random.SeedSequence(seed), (D, D_out)) / np.float32(np.sqrt(D))).astype(np.float32)

@@ -1,0 +1,66 @@
+"""bench.py host logic: the workload's FLOP counts and the replica aggregation under gloo."""
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def test_workload_flops_match_config():
+    wl = bench.workload("1.3b")
+    # 4 Nq Nk d H: full over 18 frames + chunk, local over 6 frames + chunk
+    assert wl["nq"] == 4680 and wl["nk_full"] == 32760 and wl["nk_local"] == 14040
+    assert abs(wl["flops_full"] / 1e12 - 0.942) < 5e-4
+    assert abs(wl["flops_local"] / 1e12 - 0.404) < 5e-4
+    assert wl["flops_dual"] == wl["flops_full"]
+    wl14 = bench.workload("14b")
+    assert wl14["D"] == 5120 and abs(wl14["flops_local"] / 1e12 - 1.346) < 1e-3
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    p = s.getsockname()[1]
+    s.close()
+    return p
+
+
+WORKER = r"""
+import os, sys, torch, torch.distributed as dist
+dist.init_process_group("gloo")
+r, w = dist.get_rank(), dist.get_world_size()
+# each replica reports its own time; the job's time is the max, value sums the replicas
+t = torch.tensor([10.0 + r])
+dist.all_reduce(t, op=dist.ReduceOp.MAX)
+assert t.item() == 10.0 + (w - 1)
+dist.barrier()
+if r == 0:
+    print("ok", w, t.item())
+dist.destroy_process_group()
+"""
+
+
+def test_replica_max_over_ranks_gloo(tmp_path):
+    f = tmp_path / "w.py"
+    f.write_text(WORKER)
+    env = dict(os.environ, MASTER_ADDR="127.0.0.1", MASTER_PORT=str(_free_port()))
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
+           "--master-addr=127.0.0.1", f"--master-port={env['MASTER_PORT']}", str(f)]
+    r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert "ok 2 11.0" in r.stdout
+
+
+def test_reference_arm_skips_non_zero_ranks(capsys):
+    class A:
+        model = "1.3b"
+        ref_rows = 2
+        steps = 1
+        warmup = 0
+    bench.run_reference(A, rank=1, world=2)
+    assert capsys.readouterr().out == ""

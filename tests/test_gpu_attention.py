@@ -168,3 +168,47 @@ def test_config1_sampled_rows():
     assert_close_attn(g["a_full"][rows], r["a_full"], "config1 dual full")
     assert_close_attn(g["a_loc"][rows], r["a_loc"], "config1 dual loc")
     assert np.isfinite(g["disc"]).all()
+
+
+@pytest.mark.parametrize("boost", [3.0, 6.0])
+def test_running_max_rescale_path(boost):
+    # A late frame whose keys are scaled up makes the running row max jump by more than
+    # 2^8 for some rows (boost 3: some lanes of a warp, boost 6: nearly all), exercising the
+    # lazy O rescale in TMEM, including warps where only part of the lanes need it.
+    from paper_2607_00712_gb300 import synth
+    st = Step(8, P=64, H=2, d=64, n_past=6, n_chunk_frames=2, capacity=6)
+    P = st.P
+    for f in (4, 5):
+        blk = synth.bf16_round(st.s.k_hist[f * P:(f + 1) * P] * np.float32(boost))
+        st.s.k_hist[f * P:(f + 1) * P] = blk
+        st.k_hist_res[f * P:(f + 1) * P] = blk
+        st.ring.k[:, f * P:(f + 1) * P] = bf16_tensor(blk.transpose(1, 0, 2).copy())
+    torch.cuda.synchronize()
+    _check_all_modes(st, (0, 2))
+    _check_all_modes(st, (0, 1))
+
+
+def test_back_to_back_calls_without_host_sync():
+    # Many launches queued on one stream with no host synchronisation in between (the
+    # pattern of a layer loop); results equal the single-call results bit for bit.
+    st = Step(9, P=100, H=3, d=128, n_past=9, n_chunk_frames=3, capacity=7)
+    o_ref, _ = _run_full(st)
+    l_ref, _ = _run_local(st, (0, 3))
+    g_ref = _run_dual(st, (0, 2))
+    D = st.H * st.d
+    outs = [torch.empty(st.n_q, D, dtype=torch.bfloat16, device="cuda") for _ in range(4)]
+    disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    wsb = abi.ispa_attn_dual_workspace_size(st.H, st.n_q)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    for _ in range(6):
+        abi.ispa_attn_full(st.ring.c, st.q, st.kc, st.vc, st.n_q, 0.0, outs[0])
+        abi.ispa_attn_local(st.ring.c, Window(0, 3), st.q, st.kc, st.vc, st.n_q, 0.0, outs[1])
+        abi.ispa_attn_dual(st.ring.c, Window(0, 2), st.q, st.kc, st.vc, st.n_q, 0.0, outs[2], outs[3], disc, dsum,
+                           None, None, ws, wsb)
+    torch.cuda.synchronize()
+    assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
+    assert np.array_equal(to_f32(outs[0]).reshape(o_ref.shape), o_ref)
+    assert np.array_equal(to_f32(outs[1]).reshape(l_ref.shape), l_ref)
+    assert np.array_equal(to_f32(outs[2]).reshape(o_ref.shape), g_ref["a_full"])
+    assert np.array_equal(to_f32(outs[3]).reshape(o_ref.shape), g_ref["a_loc"])
