@@ -248,6 +248,32 @@ ISPA_API ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, c
                            float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
                            ispa_stream stream);
 
+/* Largest num_heads * n_q that ispa_attn_dual_static accepts (4 MiB of fp32). */
+#define ISPA_DUAL_STATIC_MAX_PARTIALS (1u << 20)
+
+/*
+ * ispa_attn_dual without a workspace argument, for callers that cannot
+ * allocate device memory when they run the warmup pass -- e.g. a real-time
+ * streaming loop whose memory is planned once at start-up (cudaMalloc would
+ * synchronise the device mid-stream), or a plug-in whose host runtime gives it
+ * tensors but no allocator.  The paper has no counterpart; this is a library
+ * convenience.  Arguments and results are those of ispa_attn_dual.
+ *   - Scratch comes from a fixed array inside the library, present on every
+ *     GPU that loads it until the process exits; num_heads * n_q must not
+ *     exceed ISPA_DUAL_STATIC_MAX_PARTIALS, else ISPA_ERR_WORKSPACE is returned
+ *     and nothing is enqueued.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - Allocates nothing: no cudaMalloc / cudaFree, no allocating library call.
+ *   - All calls share the one array, so calls that overlap on the GPU (e.g.
+ *     on two streams) race; serialise them.  Each call overwrites every entry
+ *     it reads, so nothing needs clearing between calls.
+ */
+ISPA_API ispa_status ispa_attn_dual_static(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                                           const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                                           void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                                           float* lse_full, float* lse_loc, ispa_stream stream);
+
 /* ------------------------------------------------------------ least squares */
 
 /* Bytes of the fp32 [2*dim][2*dim] gram buffer. */

@@ -85,6 +85,8 @@ _SIGS = {
     "ispa_attn_dual": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                  c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                  c_size_t, c_void_p]),
+    "ispa_attn_dual_static": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
+                                        c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "ispa_ls_state_bytes": (c_size_t, [c_int32]),
     "ispa_ls_state_reset": (c_int32, [POINTER(LSState), c_void_p]),
     "ispa_ls_accumulate_workspace_size": (c_size_t, [c_int32, c_int64]),
@@ -210,6 +212,14 @@ def ispa_attn_dual(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: 
     _check(lib().ispa_attn_dual(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
                                 _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full),
                                 _ptr(lse_loc), _ptr(workspace), ws_bytes, _stream(stream)), "ispa_attn_dual")
+
+
+def ispa_attn_dual_static(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, a_full, a_loc,
+                          disc, disc_sq_sum, lse_full=None, lse_loc=None, stream=None) -> None:
+    """ispa_attn_dual with the library's own fixed scratch (for callers that cannot allocate)."""
+    _check(lib().ispa_attn_dual_static(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
+                                       _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full),
+                                       _ptr(lse_loc), _stream(stream)), "ispa_attn_dual_static")
 
 
 def ispa_ls_state_bytes(dim: int) -> int:
