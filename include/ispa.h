@@ -160,6 +160,12 @@ ISPA_API ispa_status ispa_debug_error_record(int32_t* rec8);
  * NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots);
 
+/* Debug aid: per-key-tile cycle trace of the attention kernel's first CTA.
+ * buf: device-accessible uint64 [n_tiles][8] (clock64 values; events 0-2 softmax
+ * S-ready / max-exchanged / P-written, 3-5 UMMA warp P-seen / PV-issued /
+ * next-S-issued, 6-7 TMA K / V issued).  NULL / 0 turns it off (the default). */
+ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
+
 /* Bytes of one ring's K and V buffers together (2 * H * cap * P * d * 2). */
 ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);
 

@@ -71,6 +71,7 @@ _SIGS = {
     "ispa_debug_wait_probe": (c_int32, [c_uint64, c_void_p]),
     "ispa_debug_error_record": (c_int32, [POINTER(c_int32)]),
     "ispa_debug_set_heartbeat": (c_int32, [c_void_p, c_int32]),
+    "ispa_debug_set_trace": (c_int32, [c_void_p, c_int32]),
     "ispa_ring_bytes": (c_size_t, [POINTER(KVRing)]),
     "ispa_ring_slot": (c_int32, [POINTER(KVRing), c_int64]),
     "ispa_window_resolve": (c_int32, [POINTER(KVRing), Window, POINTER(KeySets)]),
@@ -162,6 +163,10 @@ def ispa_debug_error_record() -> list[int]:
 
 def ispa_debug_set_heartbeat(counters, n_slots: int) -> None:
     _check(lib().ispa_debug_set_heartbeat(_ptr(counters), n_slots), "ispa_debug_set_heartbeat")
+
+
+def ispa_debug_set_trace(buf, n_tiles: int) -> None:
+    _check(lib().ispa_debug_set_trace(_ptr(buf), n_tiles), "ispa_debug_set_trace")
 
 
 def ispa_ring_bytes(ring: KVRing) -> int:

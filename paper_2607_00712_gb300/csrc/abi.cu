@@ -53,6 +53,14 @@ int g_hb_slots = 0;
 int g_hb_next = 0;
 }  // namespace
 
+uint64_t* g_trace = nullptr;
+int32_t g_trace_tiles = 0;
+
+uint64_t* trace_buffer(int32_t* n_tiles) {
+  *n_tiles = g_trace_tiles;
+  return g_trace;
+}
+
 uint32_t* next_heartbeat_slot(uint32_t kernel_tag) {
   if (!g_hb || g_hb_slots <= 0) return nullptr;
   uint32_t* slot = g_hb + 4 * (g_hb_next % g_hb_slots);
@@ -237,6 +245,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   p.status = device_status_ptr();
   if (!p.status) return ISPA_ERR_CUDA;
   p.heartbeat = next_heartbeat_slot(1);
+  p.trace = trace_buffer(&p.trace_tiles);
 
   const uint64_t row_b = static_cast<uint64_t>(HD) * 2;
   const uint64_t ring_tok = static_cast<uint64_t>(ring->capacity_frames) * P;
@@ -300,6 +309,13 @@ ispa_status ispa_last_device_error(int32_t* code) {
 ispa_status ispa_debug_error_record(int32_t* rec8) {
   if (!rec8) return ISPA_ERR_INVALID_ARG;
   if (cudaMemcpyFromSymbol(rec8, g_status, 8 * sizeof(int)) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles) {
+  if ((buf == nullptr) != (n_tiles <= 0)) return ISPA_ERR_INVALID_ARG;
+  g_trace = buf;
+  g_trace_tiles = n_tiles;
   return ISPA_OK;
 }
 

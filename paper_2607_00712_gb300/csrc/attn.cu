@@ -14,16 +14,22 @@
 // Tensor maps: the ring as (d, cap*P, H) and the chunk tensors q/k_cur/v_cur
 // as (d, H, n_q), boxes of 64 x 128 rows x 1 head with 128-byte swizzle, which
 // is the K-major (Q, K) and MN-major (V) UMMA operand layout.
-// CTA = one head x one tile of 128 queries.  Warp roles:
-//   warps 0-3  softmax: thread t of warp w owns query row 32w+t (TMEM lane);
-//   warp 4     TMA producer (Q once, then K/V tiles into staged rings);
-//   warp 5     TMEM allocator and UMMA issuer.
+// CTA = one head x one tile of 128 queries; 320 threads:
+//   warps 0-7  softmax: warp w owns query rows 32(w%4)..+31 (its TMEM lane
+//              quarter) and the score columns 64(w/4)..+63 of every key tile,
+//              so each row's 128 scores are split over two warps that swap
+//              their partial row maxima through shared memory once per tile;
+//   warp 8     TMA producer (Q once, then K/V tiles into staged rings);
+//   warp 9     TMEM allocator and UMMA issuer.
 // TMEM columns: S0 [0,128) S1 [128,256) O [256,256+d) P0 [384,448) P1 [448,512).
 // Per key tile j: S_j = Q K_j^T (SS-UMMA, fp32 in TMEM) -> softmax warps read
 // S_j, update the row max (lazy rescale of O only when the max grows by more
 // than 2^8), write P_j = exp2(.) as bf16 into TMEM -> O += P_j V_j (TS-UMMA:
 // A operand read from TMEM).  S is double buffered so S_{j+1} runs on the
 // tensor cores while the softmax warps work on S_j.
+//
+// Every wait is bounded; after a timeout the softmax warps keep executing
+// their named barriers (without touching TMEM) so no warp is left behind.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -35,14 +41,17 @@ namespace ispa {
 
 namespace {
 
-constexpr int BM = 128;       // queries per CTA
-constexpr int BN = 128;       // keys per tile
-constexpr int NTHREADS = 192;
-constexpr int WARP_TMA = 4;
-constexpr int WARP_MMA = 5;
+constexpr int BM = 128;        // queries per CTA
+constexpr int BN = 128;        // keys per tile
+constexpr int N_SOFT_WARPS = 8;
+constexpr int N_SOFT = N_SOFT_WARPS * 32;
+constexpr int NTHREADS = N_SOFT + 64;
+constexpr int WARP_TMA = 8;
+constexpr int WARP_MMA = 9;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr float RESCALE_THRESHOLD = 8.0f;  // log2 units
 constexpr uint64_t DRAIN_LIMIT_NS = 200ull * 1000 * 1000;
+constexpr int HALF_COLS = BN / 2;          // score columns per softmax warp
 
 template <int HD>
 struct Cfg {
@@ -54,10 +63,13 @@ struct Cfg {
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = TILE;
   static constexpr int OFF_V = OFF_K + KST * TILE;
-  static constexpr int OFF_BAR = OFF_V + VST * TILE;
+  static constexpr int OFF_X = OFF_V + VST * TILE;          // exchange arrays (fp32)
+  static constexpr int X_FLOATS = 2 * 2 * BM + 2 * BM + 2 * BM;  // max[2][2][BM], l[2][BM], sq[2][BM]
+  static constexpr int OFF_BAR = OFF_X + X_FLOATS * 4;
   static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
   static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16 + 1024;  // + tmem slot/abort + alignment
   static constexpr uint32_t COL_S0 = 0, COL_O = 256, COL_P0 = 384;
+  static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, HD, false, true);
 };
@@ -74,6 +86,10 @@ __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& of
   }
 }
 
+__device__ __forceinline__ void soft_barrier() {
+  asm volatile("bar.sync 1, %0;" ::"n"(N_SOFT) : "memory");
+}
+
 // Round 32 consecutive fp32 values (times inv) to bf16 pairs.
 __device__ __forceinline__ void pack_row32(const uint32_t* r, float inv, uint32_t* pk) {
 #pragma unroll
@@ -85,6 +101,29 @@ __device__ __forceinline__ void store_pk16(__nv_bfloat16* dst, const uint32_t* p
   uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
   for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+}
+
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  return static_cast<uint64_t>(__float_as_uint(a)) | (static_cast<uint64_t>(__float_as_uint(b)) << 32);
+}
+
+// (x0, x1) * c + (d, d) with one packed fp32x2 FMA
+__device__ __forceinline__ uint64_t f2_fma(uint64_t x, uint64_t c, uint64_t d) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(x), "l"(c), "l"(d));
+  return r;
+}
+
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
 }
 
 }  // namespace
@@ -99,6 +138,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
+  float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [parity][half][row]
+  float* x_l = x_max + 4 * BM;                                // [half][row]
+  float* x_sq = x_l + 2 * BM;                                 // [half][row]
   uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -135,7 +177,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b.s_full0 + 8 * i, 1);
-      mbar_init(b.p_full0 + 8 * i, BM);
+      mbar_init(b.p_full0 + 8 * i, N_SOFT);
       mbar_init(b.o_done0 + 8 * i, 1);
     }
     mbar_init(b.drain, 1);
@@ -184,6 +226,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           else tma_load_3d(sK + x * C::BOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
         }
         nk = j + 1;
+        trace_event(p.trace, p.trace_tiles, j, 6);
         if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
         mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::TILE);
         const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
@@ -193,6 +236,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           else tma_load_3d(sV + x * C::BOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
         }
         nv = j + 1;
+        trace_event(p.trace, p.trace_tiles, j, 7);
         next_tile(p, seg, off);
       }
       // Every load issued must have landed before the CTA may exit.  Older tiles of
@@ -231,6 +275,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int vs = j % C::VST;
         if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
+        trace_event(p.trace, p.trace_tiles, j, 3);
         if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
         tc_fence_after();
         const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
@@ -242,7 +287,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         tc_commit(b.o_done0 + 8 * (j & 1));
         tc_commit(b.v_empty0 + 8 * vs);
+        trace_event(p.trace, p.trace_tiles, j, 4);
         if (j + 2 < n_tiles) ok = issue_s(j + 2);
+        trace_event(p.trace, p.trace_tiles, j, 5);
       }
       // All UMMAs must have finished before TMEM is released.
       tc_commit(b.drain);
@@ -251,56 +298,68 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax warps
-    const int row = warp * 32 + lane;
+    const int quarter = warp & 3;          // TMEM lane quarter = row block
+    const int half = warp >> 2;            // score / output column half
+    const int row = quarter * 32 + lane;
     const int qrow = q0 + row;
     const bool row_ok = qrow < p.n_q;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int D = p.num_heads * HD;
     const float sl2 = p.scale_log2;
-    float m_run = -INFINITY, l_run = 0.f;
+    const uint64_t sl2x2 = f2_pack(sl2, sl2);
+    float m_run = -INFINITY, l_run = 0.f;  // l_run: this warp's column half only
     int seg = 0, off = 0;
     bool ok = true;
 
     auto warp_ok = [&](bool v) { return __all_sync(0xffffffffu, v); };
 
-    auto emit = [&](__nv_bfloat16* dst, float* lse_dst, bool with_disc) {
-      // O / l of this row -> bf16 global; optional LSE; optional discrepancy partial
-      // sum_d (A_full - A_loc)^2 of this head, taken on the stored bf16 values.
-      const float inv = 1.f / l_run;
-      __nv_bfloat16* drow = dst + static_cast<size_t>(qrow) * D + head * HD;
-      const __nv_bfloat16* lrow = p.out_loc + static_cast<size_t>(qrow) * D + head * HD;
+    // Normalise O by the full-row l and store this warp's half of the row (bf16); optional
+    // LSE; optional discrepancy partial sum_d (A_full - A_loc)^2 of this head on the stored
+    // bf16 values.  Executes the same two named barriers whether or not `live`.
+    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc) {
+      x_l[half * BM + row] = l_run;
+      soft_barrier();
+      const float l_row = l_run + x_l[(half ^ 1) * BM + row];
       float sq = 0.f;
+      if (live) {
+        const float inv = 1.f / l_row;
+        const int c0 = half * C::O_HALF;
+        __nv_bfloat16* drow = dst + static_cast<size_t>(qrow) * D + head * HD + c0;
+        const __nv_bfloat16* lrow = p.out_loc + static_cast<size_t>(qrow) * D + head * HD + c0;
 #pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(trow + C::COL_O + 32 * c, r);
-        tmem_wait_ld32(r);
-        if (row_ok) {
-          uint32_t pk[16];
-          pack_row32(r, inv, pk);
-          store_pk16(drow + 32 * c, pk);
-          if (with_disc) {
-            const uint4* l4 = reinterpret_cast<const uint4*>(lrow + 32 * c);
+        for (int c = 0; c < C::O_HALF / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(trow + C::COL_O + c0 + 32 * c, r);
+          tmem_wait_ld32(r);
+          if (row_ok) {
+            uint32_t pk[16];
+            pack_row32(r, inv, pk);
+            store_pk16(drow + 32 * c, pk);
+            if (with_disc) {
+              const uint4* l4 = reinterpret_cast<const uint4*>(lrow + 32 * c);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const uint4 v = l4[q];
-              const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+              for (int q = 0; q < 4; ++q) {
+                const uint4 v = l4[q];
+                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const uint32_t f = pk[4 * q + e];
-                const float d0 = __uint_as_float(f << 16) - __uint_as_float(w[e] << 16);
-                const float d1 = __uint_as_float(f & 0xFFFF0000u) - __uint_as_float(w[e] & 0xFFFF0000u);
-                sq = fmaf(d0, d0, sq);
-                sq = fmaf(d1, d1, sq);
+                for (int e = 0; e < 4; ++e) {
+                  const uint32_t f = pk[4 * q + e];
+                  const float d0 = __uint_as_float(f << 16) - __uint_as_float(w[e] << 16);
+                  const float d1 = __uint_as_float(f & 0xFFFF0000u) - __uint_as_float(w[e] & 0xFFFF0000u);
+                  sq = fmaf(d0, d0, sq);
+                  sq = fmaf(d1, d1, sq);
+                }
               }
             }
           }
         }
       }
-      if (row_ok) {
+      x_sq[half * BM + row] = sq;
+      soft_barrier();
+      if (live && row_ok && half == 0) {
         if (lse_dst)
-          lse_dst[static_cast<size_t>(head) * p.n_q + qrow] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
-        if (with_disc) p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = sq;
+          lse_dst[static_cast<size_t>(head) * p.n_q + qrow] = (m_run + __log2f(l_row)) * 0.69314718055994531f;
+        if (with_disc) p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = sq + x_sq[BM + row];
       }
     };
 
@@ -308,97 +367,106 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int sb = j & 1;
       if (p.dual && j == p.n_local_tiles && j > 0) {
         // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 7, j));
-        if (!ok) break;
-        tc_fence_after();
-        emit(p.out_loc, p.lse_loc, false);
+        if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 7, j));
+        if (ok) tc_fence_after();
+        emit(ok, p.out_loc, p.lse_loc, false);
       }
-      ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
-      if (!ok) break;
-      tc_fence_after();
+      if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
+      if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 0);
       const int valid = min(BN, p.seg[seg].count - off);
-      uint32_t s[BN];
-      tmem_ld32(trow + C::COL_S0 + sb * 128 + 0, s + 0);
-      tmem_ld32(trow + C::COL_S0 + sb * 128 + 32, s + 32);
-      tmem_ld32(trow + C::COL_S0 + sb * 128 + 64, s + 64);
-      tmem_ld32(trow + C::COL_S0 + sb * 128 + 96, s + 96);
-      tmem_wait_ld32(s + 0);
-      tmem_wait_ld32(s + 32);
-      tmem_wait_ld32(s + 64);
-      tmem_wait_ld32(s + 96);
-      if (valid < BN) {
-#pragma unroll
-        for (int i = 0; i < BN; ++i)
-          if (i >= valid) s[i] = __float_as_uint(-INFINITY);
-      }
-      float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < BN; i += 4) {
-        mx0 = fmaxf(mx0, __uint_as_float(s[i + 0]));
-        mx1 = fmaxf(mx1, __uint_as_float(s[i + 1]));
-        mx2 = fmaxf(mx2, __uint_as_float(s[i + 2]));
-        mx3 = fmaxf(mx3, __uint_as_float(s[i + 3]));
-      }
-      const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
-      if (j == 0) {
-        m_run = m_tile;
-      } else if (__any_sync(0xffffffffu, m_tile > m_run + RESCALE_THRESHOLD)) {
-        // Lazy rescale, decided per warp (the TMEM accesses are warp-collective):
-        // O holds PV of tiles 0..j-1 once PV_{j-1} has completed.  Lanes whose max
-        // did not grow keep alpha = 1.
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 9, j));
-        if (!ok) break;
-        tc_fence_after();
-        const float m_new = fmaxf(m_run, m_tile);
-        const float alpha = ex2_approx(m_run - m_new);
-        l_run *= alpha;
-#pragma unroll 1
-        for (int c = 0; c < HD / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(trow + C::COL_O + 32 * c, r);
-          tmem_wait_ld32(r);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-          tmem_st32(trow + C::COL_O + 32 * c, r);
-        }
-        tmem_wait_st();
-        m_run = m_new;
-      }
-      // P_j goes to TMEM buffer sb, last read by PV_{j-2}.
-      if (j >= 2) {
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc, 10, j));
-        if (!ok) break;
-        tc_fence_after();
-      }
-      const float neg_m = -m_run;
-      float rs0 = 0.f, rs1 = 0.f;
-#pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const float e0 = ex2_approx(fmaf(__uint_as_float(s[32 * c + 2 * k]), sl2, neg_m));
-          const float e1 = ex2_approx(fmaf(__uint_as_float(s[32 * c + 2 * k + 1]), sl2, neg_m));
-          rs0 += e0;
-          rs1 += e1;
-          pk[k] = pack_bf16x2(e0, e1);
-        }
-        tmem_st16(trow + C::COL_P0 + sb * 64 + 16 * c, pk);
-      }
-      l_run += rs0 + rs1;
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(b.p_full0 + 8 * sb);
-      next_tile(p, seg, off);
-    }
-    if (ok) {
-      const int jl = n_tiles - 1;
-      ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc, 11, jl));
+      uint32_t s[HALF_COLS];
+      float mx = -INFINITY;
       if (ok) {
         tc_fence_after();
-        if (p.dual && p.n_local_tiles >= n_tiles) emit(p.out_loc, p.lse_loc, false);
-        emit(p.out, p.lse, p.dual != 0);
+        const uint32_t scol = trow + C::COL_S0 + sb * 128 + half * HALF_COLS;
+        tmem_ld32(scol, s);
+        tmem_ld32(scol + 32, s + 32);
+        tmem_wait_ld32(s);
+        tmem_wait_ld32(s + 32);
+        const int vloc = valid - half * HALF_COLS;   // valid columns of this half
+        if (vloc < HALF_COLS) {
+#pragma unroll
+          for (int i = 0; i < HALF_COLS; ++i)
+            if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
+        }
+        float m0 = -INFINITY, m1 = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < HALF_COLS; i += 4) {
+          m0 = max3(m0, __uint_as_float(s[i + 0]), __uint_as_float(s[i + 1]));
+          m1 = max3(m1, __uint_as_float(s[i + 2]), __uint_as_float(s[i + 3]));
+        }
+        mx = fmaxf(m0, m1);
       }
+      x_max[(sb * 2 + half) * BM + row] = mx;
+      soft_barrier();
+      if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 1);
+      if (ok) {
+        const float m_tile = fmaxf(mx, x_max[(sb * 2 + (half ^ 1)) * BM + row]) * sl2;
+        if (j == 0) {
+          m_run = m_tile;
+        } else if (__any_sync(0xffffffffu, m_tile > m_run + RESCALE_THRESHOLD)) {
+          // Lazy rescale, decided per warp (the TMEM accesses are warp-collective; the
+          // partner warp of the same rows takes the same decision): O holds PV of tiles
+          // 0..j-1 once PV_{j-1} has completed.  Lanes whose max did not grow keep alpha = 1.
+          ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 9, j));
+          if (ok) {
+            tc_fence_after();
+            const float m_new = fmaxf(m_run, m_tile);
+            const float alpha = ex2_approx(m_run - m_new);
+            l_run *= alpha;
+#pragma unroll 1
+            for (int c = 0; c < C::O_HALF / 32; ++c) {
+              uint32_t r[32];
+              const uint32_t ocol = trow + C::COL_O + half * C::O_HALF + 32 * c;
+              tmem_ld32(ocol, r);
+              tmem_wait_ld32(r);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+              tmem_st32(ocol, r);
+            }
+            tmem_wait_st();
+            m_run = m_new;
+          }
+        }
+      }
+      // P_j goes to TMEM buffer sb, last read by PV_{j-2}.
+      if (ok && j >= 2) {
+        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc, 10, j));
+        if (ok) tc_fence_after();
+      }
+      if (ok) {
+        const uint64_t negm = f2_pack(-m_run, -m_run);
+        uint64_t acc0 = 0, acc1 = 0;
+#pragma unroll
+        for (int c = 0; c < HALF_COLS / 32; ++c) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[32 * c + 2 * k]), __uint_as_float(s[32 * c + 2 * k + 1])),
+                                      sl2x2, negm);
+            const float e0 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x)));
+            const float e1 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x >> 32)));
+            if (k & 1) acc1 = f2_add(acc1, f2_pack(e0, e1));
+            else acc0 = f2_add(acc0, f2_pack(e0, e1));
+            pk[k] = pack_bf16x2(e0, e1);
+          }
+          tmem_st16(trow + C::COL_P0 + sb * 64 + half * (HALF_COLS / 2) + 16 * c, pk);
+        }
+        const uint64_t acc = f2_add(acc0, acc1);
+        l_run += __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(b.p_full0 + 8 * sb);
+        if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 2);
+      }
+      next_tile(p, seg, off);
+    }
+    {
+      const int jl = n_tiles - 1;
+      if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc, 11, jl));
+      if (ok) tc_fence_after();
+      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
+      emit(ok, p.out, p.lse, p.dual != 0);
     }
   }
 

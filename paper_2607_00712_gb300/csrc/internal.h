@@ -41,6 +41,9 @@ struct AttnParams {
   float* disc_part;        // [H][n_q] per-head sum of squared discrepancy (dual)
   int* status;             // library status record
   uint32_t* heartbeat;     // debug counters (host-mapped) or null
+  uint64_t* trace;         // debug per-tile cycle trace of CTA (0,0) or null: [tile][8]
+  int32_t trace_tiles;
+  int32_t pad2;
 };
 
 // Launch the attention kernel.  tensor maps are encoded by the caller.
@@ -92,5 +95,6 @@ bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();
 uint32_t* next_heartbeat_slot(uint32_t kernel_tag);  // null unless a heartbeat buffer is set
+uint64_t* trace_buffer(int32_t* n_tiles);            // null unless a trace buffer is set
 
 }  // namespace ispa

@@ -111,6 +111,11 @@ __device__ __forceinline__ void heartbeat(uint32_t* hb, int idx) {
   }
 }
 
+// Debug cycle trace: tr[tile * 8 + event] = clock64() for CTA (0, 0) only.
+__device__ __forceinline__ void trace_event(uint64_t* tr, int n, int tile, int ev) {
+  if (tr && tile < n && blockIdx.x == 0 && blockIdx.y == 0) tr[tile * 8 + ev] = clock64();
+}
+
 // Drain wait used on the abort path: ignores the abort flag, fixed limit.
 __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
   const uint64_t t0 = globaltimer_ns();
