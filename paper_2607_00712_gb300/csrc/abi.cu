@@ -190,7 +190,7 @@ int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
     s.start = r[i].first_slot * P;
     s.count = r[i].n_slots * P;
     s.pad = 0;
-    tiles += (s.count + 127) / 128;
+    tiles += (s.count + kAttnBN - 1) / kAttnBN;
   }
   return tiles;
 }
@@ -228,7 +228,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
     s.src = 1;
     s.start = 0;
     s.count = n_q;
-    tiles += (n_q + 127) / 128;
+    tiles += (n_q + kAttnBN - 1) / kAttnBN;
   }
   p.n_local_tiles = tiles;
   if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P);
@@ -250,11 +250,11 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const uint64_t row_b = static_cast<uint64_t>(HD) * 2;
   const uint64_t ring_tok = static_cast<uint64_t>(ring->capacity_frames) * P;
   CUtensorMap tq, tkr, tvr, tkc, tvc;
-  bool ok = encode_tmap_3d(&tq, q, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
-            encode_tmap_3d(&tkc, k_cur, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
-            encode_tmap_3d(&tvc, v_cur, HD, H, n_q, row_b, row_b * H, 64, 1, 128) &&
-            encode_tmap_3d(&tkr, ring->k, HD, ring_tok, H, row_b, row_b * ring_tok, 64, 128, 1) &&
-            encode_tmap_3d(&tvr, ring->v, HD, ring_tok, H, row_b, row_b * ring_tok, 64, 128, 1);
+  bool ok = encode_tmap_3d(&tq, q, HD, H, n_q, row_b, row_b * H, 64, 1, kAttnBM) &&
+            encode_tmap_3d(&tkc, k_cur, HD, H, n_q, row_b, row_b * H, 64, 1, kAttnBN) &&
+            encode_tmap_3d(&tvc, v_cur, HD, H, n_q, row_b, row_b * H, 64, 1, kAttnBN) &&
+            encode_tmap_3d(&tkr, ring->k, HD, ring_tok, H, row_b, row_b * ring_tok, 64, kAttnBN, 1) &&
+            encode_tmap_3d(&tvr, ring->v, HD, ring_tok, H, row_b, row_b * ring_tok, 64, kAttnBN, 1);
   if (!ok) return ISPA_ERR_CUDA;
   if (launch_attention(HD, &tq, &tkr, &tvr, &tkc, &tvc, p, stream) != cudaSuccess) return ISPA_ERR_CUDA;
   return ISPA_OK;

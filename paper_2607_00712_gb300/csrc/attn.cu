@@ -14,19 +14,23 @@
 // Tensor maps: the ring as (d, cap*P, H) and the chunk tensors q/k_cur/v_cur
 // as (d, H, n_q), boxes of 64 x 128 rows x 1 head with 128-byte swizzle, which
 // is the K-major (Q, K) and MN-major (V) UMMA operand layout.
-// CTA = one head x one tile of 128 queries; 320 threads:
+// CTA = one head x one tile of 128 queries, key tiles of 176 keys; 320 threads:
 //   warps 0-7  softmax: warp w owns query rows 32(w%4)..+31 (its TMEM lane
-//              quarter) and the score columns 64(w/4)..+63 of every key tile,
+//              quarter) and the score columns 88(w/4)..+87 of every key tile,
 //              so each row's 128 scores are split over two warps that swap
 //              their partial row maxima through shared memory once per tile;
 //   warp 8     TMA producer (Q once, then K/V tiles into staged rings);
 //   warp 9     TMEM allocator and UMMA issuer.
-// TMEM columns: S0 [0,128) S1 [128,256) O [256,256+d) P0 [384,448) P1 [448,512).
-// Per key tile j: S_j = Q K_j^T (SS-UMMA, fp32 in TMEM) -> softmax warps read
-// S_j, update the row max (lazy rescale of O only when the max grows by more
-// than 2^8), write P_j = exp2(.) as bf16 into TMEM -> O += P_j V_j (TS-UMMA:
-// A operand read from TMEM).  S is double buffered so S_{j+1} runs on the
-// tensor cores while the softmax warps work on S_j.
+// TMEM columns: S0 [0,176) S1 [176,352) O [352,352+d).
+// Per key tile j: S_j = Q K_j^T (SS-UMMA, M=128 N=176, fp32 in TMEM) -> softmax
+// warps read S_j, update the row max (lazy rescale of O only when the max grows
+// by more than 2^8), write P_j = exp2(.) as bf16 over the first 88 columns of
+// S_j's own buffer -> O += P_j V_j (TS-UMMA: A operand read from TMEM).  S is
+// double buffered so S_{j+1} runs on the tensor cores while the softmax warps
+// work on S_j; S_{j+2} overwrites P_j only after PV_j, which the in-order
+// execution of one thread's UMMAs guarantees.  176-key tiles put more work in
+// each UMMA instruction than 128 (the per-instruction cost, not the work, bounds
+// 128x128x16 UMMAs here) while S0 + S1 + O still fit the 512 TMEM columns.
 //
 // Every wait is bounded; after a timeout the softmax warps keep executing
 // their named barriers (without touching TMEM) so no warp is left behind.
@@ -41,8 +45,8 @@ namespace ispa {
 
 namespace {
 
-constexpr int BM = 128;        // queries per CTA
-constexpr int BN = 128;        // keys per tile
+constexpr int BM = kAttnBM;    // queries per CTA
+constexpr int BN = kAttnBN;    // keys per tile
 constexpr int N_SOFT_WARPS = 8;
 constexpr int N_SOFT = N_SOFT_WARPS * 32;
 constexpr int NTHREADS = N_SOFT + 64;
@@ -52,26 +56,32 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr float RESCALE_THRESHOLD = 8.0f;  // log2 units
 constexpr uint64_t DRAIN_LIMIT_NS = 200ull * 1000 * 1000;
 constexpr int HALF_COLS = BN / 2;          // score columns per softmax warp
+constexpr int P_HALF = HALF_COLS / 2;      // packed bf16 P columns per softmax warp
+static_assert(BN % 16 == 0 && BN <= 256 && HALF_COLS % 8 == 0 && P_HALF % 4 == 0, "key tile shape");
 
 template <int HD>
 struct Cfg {
   static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per tile row
-  static constexpr int BOX = 128 * 128;         // [128 rows][64 bf16] = 16 KB
-  static constexpr int TILE = NBOX * BOX;       // one Q, K or V tile
-  static constexpr int KST = HD == 128 ? 3 : 4;  // K stages
+  static constexpr int QBOX = BM * 128;         // [128 rows][64 bf16] = 16 KB
+  static constexpr int KBOX = BN * 128;         // [176 rows][64 bf16] = 22 KB
+  static constexpr int Q_TILE = NBOX * QBOX;
+  static constexpr int KV_TILE = NBOX * KBOX;   // one K or V tile
+  static constexpr int KST = HD == 128 ? 2 : 4;  // K stages
   static constexpr int VST = HD == 128 ? 2 : 4;  // V stages
   static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = TILE;
-  static constexpr int OFF_V = OFF_K + KST * TILE;
-  static constexpr int OFF_X = OFF_V + VST * TILE;          // exchange arrays (fp32)
+  static constexpr int OFF_K = Q_TILE;
+  static constexpr int OFF_V = OFF_K + KST * KV_TILE;
+  static constexpr int OFF_X = OFF_V + VST * KV_TILE;          // exchange arrays (fp32)
   static constexpr int X_FLOATS = 2 * 2 * BM + 2 * BM + 2 * BM;  // max[2][2][BM], l[2][BM], sq[2][BM]
   static constexpr int OFF_BAR = OFF_X + X_FLOATS * 4;
   static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
   static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16 + 1024;  // + tmem slot/abort + alignment
-  static constexpr uint32_t COL_S0 = 0, COL_O = 256, COL_P0 = 384;
+  static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
   static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, HD, false, true);
+  static_assert(COL_O + HD <= 512, "TMEM columns");
+  static_assert(KBOX % 1024 == 0 && QBOX % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
 };
 
 struct Bars {
@@ -208,9 +218,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       const uint32_t sQ = sbase + C::OFF_Q;
-      mbar_arrive_expect_tx(b.q_full, C::TILE);
+      mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
 #pragma unroll
-      for (int x = 0; x < C::NBOX; ++x) tma_load_3d(sQ + x * C::BOX, &tm_q, b.q_full, 64 * x, head, q0);
+      for (int x = 0; x < C::NBOX; ++x) tma_load_3d(sQ + x * C::QBOX, &tm_q, b.q_full, 64 * x, head, q0);
       int seg = 0, off = 0;
       int nk = 0, nv = 0;  // K and V tiles issued
       for (int j = 0; j < n_tiles; ++j) {
@@ -218,22 +228,22 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int row = p.seg[seg].start + off;
         const int ks = j % C::KST, vs = j % C::VST;
         if (!mbar_wait(b.k_empty0 + 8 * ks, ((j / C::KST) & 1) ^ 1, wc, 1, j)) break;
-        mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::TILE);
-        const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
+        mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::KV_TILE);
+        const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
 #pragma unroll
         for (int x = 0; x < C::NBOX; ++x) {
-          if (chunk) tma_load_3d(sK + x * C::BOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
-          else tma_load_3d(sK + x * C::BOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
+          if (chunk) tma_load_3d(sK + x * C::KBOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
+          else tma_load_3d(sK + x * C::KBOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
         }
         nk = j + 1;
         trace_event(p.trace, p.trace_tiles, j, 6);
         if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
-        mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::TILE);
-        const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
+        mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::KV_TILE);
+        const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
 #pragma unroll
         for (int x = 0; x < C::NBOX; ++x) {
-          if (chunk) tma_load_3d(sV + x * C::BOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
-          else tma_load_3d(sV + x * C::BOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
+          if (chunk) tma_load_3d(sV + x * C::KBOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
+          else tma_load_3d(sV + x * C::KBOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
         }
         nv = j + 1;
         trace_event(p.trace, p.trace_tiles, j, 7);
@@ -258,13 +268,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int ks = j % C::KST;
         if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc, 4, j)) return false;
         tc_fence_after();
-        const uint32_t sK = sbase + C::OFF_K + ks * C::TILE;
-        const uint32_t d = tmem + C::COL_S0 + (j & 1) * 128;
+        const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
+        const uint32_t d = tmem + C::COL_S0 + (j & 1) * BN;
 #pragma unroll
         for (int k = 0; k < HD / 16; ++k) {
-          const uint32_t koff = (k >> 2) * C::BOX + (k & 3) * 32;
-          umma_ss(d, sw128_desc(sQ + koff, 16, 1024), sw128_desc(sK + koff, 16, 1024), C::IDESC_QK,
-                  k > 0 ? 1u : 0u);
+          const uint32_t kin = (k & 3) * 32;
+          umma_ss(d, sw128_desc(sQ + (k >> 2) * C::QBOX + kin, 16, 1024),
+                  sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
         }
         tc_commit(b.s_full0 + 8 * (j & 1));
         tc_commit(b.k_empty0 + 8 * ks);
@@ -278,11 +288,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         trace_event(p.trace, p.trace_tiles, j, 3);
         if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
         tc_fence_after();
-        const uint32_t sV = sbase + C::OFF_V + vs * C::TILE;
-        const uint32_t a = tmem + C::COL_P0 + (j & 1) * 64;
+        const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
+        const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
 #pragma unroll
         for (int k = 0; k < BN / 16; ++k) {
-          umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::BOX, 1024), C::IDESC_PV,
+          umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::KBOX, 1024), C::IDESC_PV,
                   (j > 0 || k > 0) ? 1u : 0u);
         }
         tc_commit(b.o_done0 + 8 * (j & 1));
@@ -378,11 +388,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       float mx = -INFINITY;
       if (ok) {
         tc_fence_after();
-        const uint32_t scol = trow + C::COL_S0 + sb * 128 + half * HALF_COLS;
-        tmem_ld32(scol, s);
-        tmem_ld32(scol + 32, s + 32);
-        tmem_wait_ld32(s);
-        tmem_wait_ld32(s + 32);
+        const uint32_t scol = trow + C::COL_S0 + sb * BN + half * HALF_COLS;
+#pragma unroll
+        for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
+#pragma unroll
+        for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
         const int vloc = valid - half * HALF_COLS;   // valid columns of this half
         if (vloc < HALF_COLS) {
 #pragma unroll
@@ -429,28 +439,27 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
         }
       }
-      // P_j goes to TMEM buffer sb, last read by PV_{j-2}.
-      if (ok && j >= 2) {
-        ok = warp_ok(mbar_wait(b.o_done0 + 8 * sb, ((j - 2) >> 1) & 1, wc, 10, j));
-        if (ok) tc_fence_after();
-      }
+      // P_j overwrites S_j in buffer sb: both halves have copied their S columns out
+      // (the max exchange above is a barrier), and PV_{j-2}, the last reader of this
+      // buffer's previous P, precedes S_j in the UMMA stream.
       if (ok) {
         const uint64_t negm = f2_pack(-m_run, -m_run);
         uint64_t acc0 = 0, acc1 = 0;
+        const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
 #pragma unroll
-        for (int c = 0; c < HALF_COLS / 32; ++c) {
-          uint32_t pk[16];
+        for (int c = 0; c < P_HALF / 4; ++c) {
+          uint32_t pk[4];
 #pragma unroll
-          for (int k = 0; k < 16; ++k) {
-            const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[32 * c + 2 * k]), __uint_as_float(s[32 * c + 2 * k + 1])),
-                                      sl2x2, negm);
+          for (int k = 0; k < 4; ++k) {
+            const int e = 8 * c + 2 * k;
+            const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), sl2x2, negm);
             const float e0 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x)));
             const float e1 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x >> 32)));
             if (k & 1) acc1 = f2_add(acc1, f2_pack(e0, e1));
             else acc0 = f2_add(acc0, f2_pack(e0, e1));
             pk[k] = pack_bf16x2(e0, e1);
           }
-          tmem_st16(trow + C::COL_P0 + sb * 64 + half * (HALF_COLS / 2) + 16 * c, pk);
+          tmem_st4(pcol + 4 * c, pk);
         }
         const uint64_t acc = f2_add(acc0, acc1);
         l_run += __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
