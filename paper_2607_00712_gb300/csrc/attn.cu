@@ -221,33 +221,45 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
 #pragma unroll
       for (int x = 0; x < C::NBOX; ++x) tma_load_3d(sQ + x * C::QBOX, &tm_q, b.q_full, 64 * x, head, q0);
-      int seg = 0, off = 0;
+      // Loads are issued in the order their stages free up: the UMMA stream is
+      // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so stages free as K_t (after S_{t-KST}) then
+      // V_{t-1} (after PV_{t-1-VST}); V therefore trails K by one tile.
+      int kseg = 0, koff = 0, vseg = 0, voff = 0;
       int nk = 0, nv = 0;  // K and V tiles issued
-      for (int j = 0; j < n_tiles; ++j) {
-        const bool chunk = p.seg[seg].src != 0;
-        const int row = p.seg[seg].start + off;
-        const int ks = j % C::KST, vs = j % C::VST;
-        if (!mbar_wait(b.k_empty0 + 8 * ks, ((j / C::KST) & 1) ^ 1, wc, 1, j)) break;
-        mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::KV_TILE);
-        const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
+      for (int t = 0; t <= n_tiles; ++t) {
+        if (t < n_tiles) {
+          const bool chunk = p.seg[kseg].src != 0;
+          const int row = p.seg[kseg].start + koff;
+          const int ks = t % C::KST;
+          if (!mbar_wait(b.k_empty0 + 8 * ks, ((t / C::KST) & 1) ^ 1, wc, 1, t)) break;
+          mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::KV_TILE);
+          const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
 #pragma unroll
-        for (int x = 0; x < C::NBOX; ++x) {
-          if (chunk) tma_load_3d(sK + x * C::KBOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
-          else tma_load_3d(sK + x * C::KBOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
+          for (int x = 0; x < C::NBOX; ++x) {
+            if (chunk) tma_load_3d(sK + x * C::KBOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
+            else tma_load_3d(sK + x * C::KBOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
+          }
+          nk = t + 1;
+          trace_event(p.trace, p.trace_tiles, t, 6);
+          next_tile(p, kseg, koff);
         }
-        nk = j + 1;
-        trace_event(p.trace, p.trace_tiles, j, 6);
-        if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
-        mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::KV_TILE);
-        const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
+        if (t >= 1) {
+          const int j = t - 1;
+          const bool chunk = p.seg[vseg].src != 0;
+          const int row = p.seg[vseg].start + voff;
+          const int vs = j % C::VST;
+          if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
+          mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::KV_TILE);
+          const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
 #pragma unroll
-        for (int x = 0; x < C::NBOX; ++x) {
-          if (chunk) tma_load_3d(sV + x * C::KBOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
-          else tma_load_3d(sV + x * C::KBOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
+          for (int x = 0; x < C::NBOX; ++x) {
+            if (chunk) tma_load_3d(sV + x * C::KBOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
+            else tma_load_3d(sV + x * C::KBOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
+          }
+          nv = j + 1;
+          trace_event(p.trace, p.trace_tiles, j, 7);
+          next_tile(p, vseg, voff);
         }
-        nv = j + 1;
-        trace_event(p.trace, p.trace_tiles, j, 7);
-        next_tile(p, seg, off);
       }
       // Every load issued must have landed before the CTA may exit.  Older tiles of
       // a stage completed before the stage was refilled, so the last KST (VST) suffice.
