@@ -49,6 +49,19 @@ def log(*a):
     print(*a, file=sys.stderr, flush=True)
 
 
+# DRAM bytes of one F-layer attention launch of the 1.3B step (dram__bytes_read.sum +
+# dram__bytes_write.sum from one ncu capture, profiles/attn_kernel_1.3b_chunk_step.md), valid
+# only for the kernel source it was taken on: reported as null once attn.cu / ptx.cuh change.
+ATTN_TRAFFIC = {"source_sha256_16": "6316d396fd49e0ed", "bytes": 242547200 + 12269824, "model": "1.3b"}
+
+
+def attn_source_sha():
+    import hashlib
+    d = os.path.join(ROOT, "paper_2607_00712_gb300", "csrc")
+    src = open(os.path.join(d, "attn.cu"), "rb").read() + open(os.path.join(d, "ptx.cuh"), "rb").read()
+    return hashlib.sha256(src).hexdigest()[:16]
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -283,8 +296,11 @@ def run_ours(args, rank, world, local_rank):
             if isinstance(v_, float):
                 m[k_] = round(v_, 4)
     achieved = modes["full"]["tflops"]
+    traffic = None
+    if ATTN_TRAFFIC["model"] == args.model and attn_source_sha() == ATTN_TRAFFIC["source_sha256_16"]:
+        traffic = ATTN_TRAFFIC["bytes"]
     roofline = dict(bound="tensor", achieved=round(achieved, 2), peak=pk["bf16"], unit="TFLOP/s",
-                    frac=round(achieved / pk["bf16"], 4), traffic=None,
+                    frac=round(achieved / pk["bf16"], 4), traffic=traffic, traffic_unit="bytes per launch",
                     kernel="attn_kernel<128> (F-layer launch)", peak_source=pk["source"] + " burst bf16",
                     frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
 
