@@ -305,6 +305,8 @@ def run_ours(args, rank, world, local_rank):
                     frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
 
     log(f"[bench] timed steps done at {time.perf_counter() - t_start:.1f} s")
+    extras = run_extras(r, wl, device)
+    log(f"[bench] extras done at {time.perf_counter() - t_start:.1f} s")
     e2e = run_e2e(r, args, device, flops_step, world)
     log(f"[bench] e2e done at {time.perf_counter() - t_start:.1f} s")
 
@@ -315,13 +317,68 @@ def run_ours(args, rank, world, local_rank):
                               heads=wl["H"], head_dim=wl["d"], tokens_per_frame=wl["P"], n_q=wl["nq"],
                               f_ring_frames=wl["F"], window_frames=wl["W"], parallelism=f"replicas x{world}",
                               l2="flushed between steps (256 MB write outside timed events)"),
-                  modes=modes, roofline=roofline, e2e=e2e,
+                  modes=modes, roofline=roofline, e2e=e2e, extras=extras,
                   gpu_launches=r.launches_per_step * args.steps, clocks=clocks,
                   wall_s=round(wall, 3))
     if rank == 0:
         if args.cpu_baseline:
             result["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_rows)
         print(json.dumps(result), flush=True)
+
+
+def run_extras(r, wl, device, reps=20):
+    """Once-per-run figures outside the step: the paper's two-call dual pass (Eq. 9-12: local
+    branch, history branch, LSE merge) against the fused one-sweep dual kernel, and the
+    closed-form solve (Eq. 5-6) of the accumulated state."""
+    import torch
+    abi = r.abi
+    nq, H, d, D = wl["nq"], wl["H"], wl["d"], wl["D"]
+    q, kc, vc = r.inputs[2]
+    ring = r.rings[2].c
+    o_loc = torch.empty(nq, D, dtype=torch.bfloat16, device=device)
+    o_hist = torch.empty_like(o_loc)
+    fused = torch.empty_like(o_loc)
+    l_loc = torch.empty(H, nq, dtype=torch.float32, device=device)
+    l_hist = torch.empty_like(l_loc)
+    l_out = torch.empty_like(l_loc)
+    s = r.stream
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    t_loc = t_hist = t_merge = t_dual = 0.0
+    for _ in range(reps):
+        ev[0].record(s)
+        abi.ispa_attn_local(ring, r.win, q, kc, vc, nq, 0.0, o_loc, l_loc, s)
+        ev[1].record(s)
+        abi.ispa_attn_hist(ring, r.win, q, nq, 0.0, o_hist, l_hist, s)
+        ev[2].record(s)
+        abi.ispa_lse_merge(o_loc, l_loc, o_hist, l_hist, nq, H, d, fused, l_out, s)
+        ev[3].record(s)
+        abi.ispa_attn_dual(ring, r.win, q, kc, vc, nq, 0.0, r.a_full, r.a_loc, r.disc, r.disc_sum, None, None,
+                           r.dual_ws, r.dual_wsb, s)
+        ev[4].record(s)
+        torch.cuda.synchronize(device)
+        t_loc += ev[0].elapsed_time(ev[1])
+        t_hist += ev[1].elapsed_time(ev[2])
+        t_merge += ev[2].elapsed_time(ev[3])
+        t_dual += ev[3].elapsed_time(ev[4])
+    dec = (t_loc + t_hist + t_merge) / reps
+    out = dict(decomposed_dual_ms=round(dec, 4), fused_dual_ms=round(t_dual / reps, 4),
+               decomposed_merge_ms=round(t_merge / reps, 4),
+               merge_share_of_decomposed=round(t_merge / reps / dec, 4))
+    # closed-form solve of the accumulated state (once per transition)
+    from paper_2607_00712_gb300 import synth
+    W = torch.from_numpy(synth.make_weight(1, D, D)).to(device)
+    dW = torch.empty(D, D, dtype=torch.float32, device=device)
+    wsb = abi.ispa_ls_solve_workspace_size(D, D)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=device)
+    torch.cuda.synchronize(device)
+    t0 = time.perf_counter()
+    try:
+        abi.ispa_ls_solve(r.ls.c, W, D, 1e-3, dW, ws, wsb, s)
+        out["ls_solve_ms"] = round((time.perf_counter() - t0) * 1e3, 2)
+        out["ls_solve_dim"] = D
+    except abi.IspaError as e:
+        out["ls_solve_error"] = str(e)
+    return out
 
 
 def run_e2e(r, args, device, flops_step, world):
@@ -428,7 +485,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--model", choices=sorted(MODELS), default="1.3b")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--cpu-sample-rows", type=int, default=128)
+    ap.add_argument("--cpu-sample-rows", type=int, default=1024)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--watchdog", type=float, default=300.0, help="dump Python stacks after this many s")
     args = ap.parse_args()

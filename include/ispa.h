@@ -280,6 +280,64 @@ ISPA_API ispa_status ispa_attn_dual_static(const ispa_kv_ring* ring, ispa_window
                                            void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
                                            float* lse_full, float* lse_loc, ispa_stream stream);
 
+/*
+ * History branch of the decomposed dual pass (Eq. 10): attention of the chunk's
+ * queries over the history set only -- the resident past frames outside the
+ * window, without the chunk.  Together with ispa_attn_local (Eq. 9) and
+ * ispa_lse_merge (Eq. 11-12) it is the paper's two-call form of the dual pass;
+ * ispa_attn_dual computes the same in one sweep.  Arguments as for
+ * ispa_attn_local; lse must not be NULL here.  An empty history set gives
+ * out = 0 and lse = -inf (a branch that contributes nothing to the merge).
+ */
+ISPA_API ispa_status ispa_attn_hist(const ispa_kv_ring* ring, ispa_window win, const void* q, int32_t n_q,
+                                    float scale, void* out, float* lse, ispa_stream stream);
+
+/*
+ * Eq. 11-12: merge two attention branches over disjoint key sets.
+ *   o_a, o_b   : bf16 [n_q][num_heads * head_dim]; lse_a, lse_b : fp32 [num_heads][n_q]
+ *   out        : bf16 [n_q][num_heads * head_dim]; lse_out : fp32 [num_heads][n_q] or NULL
+ * LSE = log(exp(lse_a) + exp(lse_b)); out = exp(lse_a - LSE) o_a + exp(lse_b - LSE) o_b,
+ * in fp32, rounded to bf16.  A branch with lse = -inf has weight 0.  out may alias o_a or o_b.
+ */
+ISPA_API ispa_status ispa_lse_merge(const void* o_a, const float* lse_a, const void* o_b, const float* lse_b,
+                                    int32_t n_q, int32_t num_heads, int32_t head_dim, void* out, float* lse_out,
+                                    ispa_stream stream);
+
+/* ------------------------------------------------------------ transition */
+
+/*
+ * Host-only dynamic layer selection (Sec. 3.3): rank the n_layers layers by
+ * ascending feasibility score eps (host array) and mark the k lowest as
+ * L-layers (is_l_layer[i] = 1, else 0; host array of n_layers).  Ties go to
+ * the lower layer index; NaN scores rank last.  0 <= k <= n_layers.
+ */
+ISPA_API ispa_status ispa_select_layers(const double* eps, int32_t n_layers, int32_t k, int32_t* is_l_layer);
+
+/*
+ * Weight injection W_new = W + dW (Sec. 3.1 phase 3, Sec. 3.3), in place, on
+ * the output projection in row-vector convention.
+ *   W  : fp32 [dim][d_out] (ispa_apply_absorption) or bf16 (..._bf16: the sum is
+ *        taken in fp32 and rounded to bf16);  dW : fp32 [dim][d_out].
+ */
+ISPA_API ispa_status ispa_apply_absorption(float* W, const float* dW, int32_t dim, int32_t d_out,
+                                           ispa_stream stream);
+ISPA_API ispa_status ispa_apply_absorption_bf16(void* W, const float* dW, int32_t dim, int32_t d_out,
+                                                ispa_stream stream);
+
+/*
+ * Permanent eviction of an L-layer's history (Sec. 3.1 phase 3: "completely
+ * discard their historical KV cache, retaining only the local context"): copy
+ * the window's frames of `src` into the smaller caller-allocated ring `dst`
+ * and make dst the layer's cache.  dst must have src's head shape,
+ * n_sink_frames == win.n_sink_frames and capacity_frames == win.n_sink_frames +
+ * win.n_recent_frames; on success dst->frames_written = src->frames_written and
+ * every frame of the window sits in its dst slot (so later appends keep the
+ * window sliding).  Errors: ISPA_ERR_CAPACITY if a window frame is not resident
+ * in src, ISPA_ERR_INVALID_ARG on mismatched shapes.
+ */
+ISPA_API ispa_status ispa_ring_compact(const ispa_kv_ring* src, ispa_window win, ispa_kv_ring* dst,
+                                       ispa_stream stream);
+
 /* ------------------------------------------------------------ least squares */
 
 /* Bytes of the fp32 [2*dim][2*dim] gram buffer. */

@@ -17,6 +17,8 @@ past frames has past frames 0..F-1; the chunk is not part of the cache.
 """
 from __future__ import annotations
 
+import math
+
 
 def local_past_frames(F: int, n_sink: int, n_recent: int) -> list[int]:
     """Past frames in the local set: {f < n_sink} united with {F-n_recent <= f < F}."""
@@ -65,6 +67,18 @@ def slot_ranges(frames: list[int], capacity: int, n_pinned: int) -> list[tuple[i
         else:
             runs.append((s, 1))
     return runs
+
+
+def select_layers(eps, k: int) -> list[int]:
+    """Sec. 3.3: rank layers by ascending feasibility score and pick the k lowest as L-layers.
+
+    Returns a 0/1 list (1 = L-layer).  Ties keep the lower layer index first (the paper
+    gives only "ascending order"); a NaN score ranks after every number.
+    """
+    n = len(eps)
+    key = [(1 if math.isnan(e) else 0, 0.0 if math.isnan(e) else e, i) for i, e in enumerate(eps)]
+    chosen = [i for _, _, i in sorted(key)[:k]]
+    return [1 if i in chosen else 0 for i in range(n)]
 
 
 def ring_bytes(num_heads: int, head_dim: int, tokens_per_frame: int,

@@ -88,6 +88,13 @@ _SIGS = {
                                  c_size_t, c_void_p]),
     "ispa_attn_dual_static": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                         c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_hist": (c_int32, [POINTER(KVRing), Window, c_void_p, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
+    "ispa_lse_merge": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p,
+                                 c_void_p]),
+    "ispa_select_layers": (c_int32, [POINTER(c_double), c_int32, c_int32, POINTER(c_int32)]),
+    "ispa_apply_absorption": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p]),
+    "ispa_apply_absorption_bf16": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p]),
+    "ispa_ring_compact": (c_int32, [POINTER(KVRing), Window, POINTER(KVRing), c_void_p]),
     "ispa_ls_state_bytes": (c_size_t, [c_int32]),
     "ispa_ls_state_reset": (c_int32, [POINTER(LSState), c_void_p]),
     "ispa_ls_accumulate_workspace_size": (c_size_t, [c_int32, c_int64]),
@@ -225,6 +232,38 @@ def ispa_attn_dual_static(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, 
     _check(lib().ispa_attn_dual_static(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
                                        _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full),
                                        _ptr(lse_loc), _stream(stream)), "ispa_attn_dual_static")
+
+
+def ispa_attn_hist(ring: KVRing, win: Window, q, n_q: int, scale: float, out, lse, stream=None) -> None:
+    _check(lib().ispa_attn_hist(ctypes.byref(ring), win, _ptr(q), n_q, scale, _ptr(out), _ptr(lse), _stream(stream)),
+           "ispa_attn_hist")
+
+
+def ispa_lse_merge(o_a, lse_a, o_b, lse_b, n_q: int, num_heads: int, head_dim: int, out, lse_out=None,
+                   stream=None) -> None:
+    _check(lib().ispa_lse_merge(_ptr(o_a), _ptr(lse_a), _ptr(o_b), _ptr(lse_b), n_q, num_heads, head_dim, _ptr(out),
+                                _ptr(lse_out), _stream(stream)), "ispa_lse_merge")
+
+
+def ispa_select_layers(eps, k: int) -> list[int]:
+    n = len(eps)
+    e = (c_double * n)(*eps)
+    out = (c_int32 * n)()
+    _check(lib().ispa_select_layers(e, n, k, out), "ispa_select_layers")
+    return list(out)
+
+
+def ispa_apply_absorption(W, dW, dim: int, d_out: int, stream=None) -> None:
+    _check(lib().ispa_apply_absorption(_ptr(W), _ptr(dW), dim, d_out, _stream(stream)), "ispa_apply_absorption")
+
+
+def ispa_apply_absorption_bf16(W, dW, dim: int, d_out: int, stream=None) -> None:
+    _check(lib().ispa_apply_absorption_bf16(_ptr(W), _ptr(dW), dim, d_out, _stream(stream)),
+           "ispa_apply_absorption_bf16")
+
+
+def ispa_ring_compact(src: KVRing, win: Window, dst: KVRing, stream=None) -> None:
+    _check(lib().ispa_ring_compact(ctypes.byref(src), win, ctypes.byref(dst), _stream(stream)), "ispa_ring_compact")
 
 
 def ispa_ls_state_bytes(dim: int) -> int:

@@ -180,7 +180,7 @@ ispa_status resolve(const ispa_kv_ring* r, ispa_window win, ispa_key_sets* ks) {
 }
 
 // ------------------------------------------------------------ attention driver
-enum Mode { MODE_FULL, MODE_LOCAL, MODE_DUAL };
+enum Mode { MODE_FULL, MODE_LOCAL, MODE_DUAL, MODE_HIST };
 
 int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
   int tiles = 0;
@@ -218,21 +218,29 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const ispa_slot_range chunk{0, 0};
   (void)chunk;
   int tiles = 0;
-  if (mode == MODE_FULL) {
+  if (mode == MODE_HIST) {
+    // Eq. 10: the history set alone, no chunk
+    tiles = add_segs(p, 0, ks.hist, ks.n_hist, P);
+    if (tiles == 0) return launch_empty_branch(out, lse, n_q, H, HD, stream) == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
+    p.n_local_tiles = tiles;
+    p.n_tiles = tiles;
+  } else if (mode == MODE_FULL) {
     tiles += add_segs(p, 0, ks.full, ks.n_full, P);
   } else {
     tiles += add_segs(p, 0, ks.local, ks.n_local, P);
   }
-  {
+  if (mode != MODE_HIST) {
     AttnSeg& s = p.seg[p.n_seg++];
     s.src = 1;
     s.start = 0;
     s.count = n_q;
     tiles += (n_q + kAttnBN - 1) / kAttnBN;
   }
-  p.n_local_tiles = tiles;
-  if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P);
-  p.n_tiles = tiles;
+  if (mode != MODE_HIST) {
+    p.n_local_tiles = tiles;
+    if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P);
+    p.n_tiles = tiles;
+  }
   p.dual = mode == MODE_DUAL ? 1 : 0;
   const float sc = scale == 0.f ? 1.f / sqrtf(static_cast<float>(HD)) : scale;
   p.scale_log2 = sc * 1.4426950408889634f;
@@ -418,6 +426,13 @@ ispa_status ispa_attn_local(const ispa_kv_ring* ring, ispa_window win, const voi
                             void* out, float* lse, ispa_stream stream) {
   return attn_common(MODE_LOCAL, ring, win, q, k_cur, v_cur, n_q, scale, out, nullptr, lse, nullptr,
                      nullptr, stream);
+}
+
+ispa_status ispa_attn_hist(const ispa_kv_ring* ring, ispa_window win, const void* q, int32_t n_q, float scale,
+                           void* out, float* lse, ispa_stream stream) {
+  if (!lse) return ISPA_ERR_INVALID_ARG;
+  // the chunk tensors are not read in this mode; q stands in for them in the unused maps
+  return attn_common(MODE_HIST, ring, win, q, q, q, n_q, scale, out, nullptr, lse, nullptr, nullptr, stream);
 }
 
 size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q) {

@@ -56,6 +56,9 @@ cudaError_t launch_attention(int head_dim, const CUtensorMap* tm_q, const CUtens
 cudaError_t launch_disc_reduce(const float* part, int32_t H, int32_t n_q, float* disc,
                                float* disc_sq_sum, cudaStream_t s);
 
+// O = 0 and LSE = -inf for an empty key set (the history branch with no history).
+cudaError_t launch_empty_branch(void* out, float* lse, int32_t n_q, int32_t H, int32_t d, cudaStream_t s);
+
 // ------------------------------------------------------------ KV append
 constexpr int kMaxAppendFrames = 16;
 constexpr int kMaxAppendLayers = 64;

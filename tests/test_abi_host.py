@@ -147,3 +147,26 @@ def test_workspace_sizes():
     assert abi.ispa_ls_state_bytes(1536) == 4 * 1536 * 1536 * 4
     assert abi.ispa_ls_accumulate_workspace_size(1536, 4680) >= 2 * 4680 * 1536 * 2
     assert abi.ispa_ls_solve_workspace_size(1536, 1536) >= 3 * 1536 * 1536 * 8
+
+
+def test_select_layers_matches_oracle():
+    import random
+    rnd = random.Random(5)
+    for _ in range(40):
+        n = rnd.randint(1, 40)
+        eps = [rnd.choice([0.25, 1.0, rnd.random(), float("nan")]) for _ in range(n)]
+        k = rnd.randint(0, n)
+        assert abi.ispa_select_layers(eps, k) == ks.select_layers(eps, k)
+    with pytest.raises(abi.IspaError):
+        abi.ispa_select_layers([1.0, 2.0], 3)
+
+
+def test_ring_compact_validation_without_gpu():
+    L = abi.lib()
+    src = KVRing(2, 64, 16, 10, 0, 0, 13, 16, 16)
+    dst = KVRing(2, 64, 16, 5, 1, 0, 0, 16, 16)          # wrong capacity for window (1, 3)
+    assert L.ispa_ring_compact(ctypes.byref(src), Window(1, 3), ctypes.byref(dst), None) == abi.ISPA_ERR_INVALID_ARG
+    dst = KVRing(2, 64, 16, 4, 1, 0, 0, 16, 16)
+    # frame 0 (the sink) was evicted from src (no pinned sink there): the window cannot be kept
+    assert L.ispa_ring_compact(ctypes.byref(src), Window(1, 3), ctypes.byref(dst), None) == abi.ISPA_ERR_CAPACITY
+    assert dst.frames_written == 0

@@ -101,3 +101,26 @@ def test_slot_ranges_wrap():
 def test_ring_bytes():
     # config "1.3B": 12 heads x 128 x 1560 tokens, 18 frames, K and V, bf16
     assert ks.ring_bytes(12, 128, 1560, 18) == 2 * 12 * 18 * 1560 * 128 * 2
+
+
+def test_select_layers_ascending_with_ties_and_nan():
+    # Sec. 3.3: the k layers with the lowest eps become L-layers.
+    eps = [3.0, 1.0, float("nan"), 1.0, 0.5, 7.0]
+    assert ks.select_layers(eps, 0) == [0, 0, 0, 0, 0, 0]
+    assert ks.select_layers(eps, 1) == [0, 0, 0, 0, 1, 0]
+    assert ks.select_layers(eps, 2) == [0, 1, 0, 0, 1, 0]      # tie 1.0: lower index first
+    assert ks.select_layers(eps, 3) == [0, 1, 0, 1, 1, 0]
+    assert ks.select_layers(eps, 6) == [1, 1, 1, 1, 1, 1]
+    assert ks.select_layers(eps, 5) == [1, 1, 0, 1, 1, 1]      # NaN last
+
+
+def test_select_layers_matches_sort_brute_force():
+    import random
+    rnd = random.Random(3)
+    for _ in range(50):
+        n = rnd.randint(1, 12)
+        eps = [rnd.choice([0.0, 1.0, 2.0, rnd.random()]) for _ in range(n)]
+        k = rnd.randint(0, n)
+        want = sorted(range(n), key=lambda i: (eps[i], i))[:k]
+        got = ks.select_layers(eps, k)
+        assert [i for i in range(n) if got[i]] == sorted(want)
