@@ -56,8 +56,8 @@ typedef enum {
 } ispa_status;
 
 /*
- * Per-layer KV cache as a frame-granular ring (Sec. 2: "truncated to include
- * only the KV pairs from the most recent frames"; Sec. 3.4: sink frame K_1).
+ * Per-layer KV cache as a frame-granular ring (Sec. 2: the cache keeps only
+ * the latest frames' keys and values; Sec. 3.4: the sink frame K_1 is kept).
  *   k, v : bf16 [num_heads][capacity_frames * tokens_per_frame][head_dim],
  *          caller-owned device memory of ispa_ring_bytes()/2 bytes each.
  *   Logical frame f (0, 1, 2, ... in generation order) lives in slot
@@ -68,7 +68,9 @@ typedef enum {
  *   overwrites the oldest non-sink frame.  frames_written counts the frames
  *   appended so far; it is advanced on the host by ispa_kv_append when the
  *   copy is enqueued.  The struct is plain data: copying it (and the two
- *   buffers) checkpoints the cache.
+ *   buffers) checkpoints the cache.  Slots never written must still hold
+ *   finite values (zero-fill the buffers at creation): a key tile that ends
+ *   inside a run reads the rows after it with weight zero, and 0 * NaN is NaN.
  */
 typedef struct {
   int32_t num_heads;
@@ -133,8 +135,10 @@ typedef struct {
 ISPA_API const char* ispa_status_string(ispa_status s);
 
 /* Device error recorded by a kernel on the current device since the last
- * call (then cleared): ISPA_OK or ISPA_ERR_TIMEOUT.  Synchronises the device
- * with a blocking copy of one word.  *code (nullable, host) gets the raw code. */
+ * call (then cleared): ISPA_OK, ISPA_ERR_TIMEOUT (raw code 1), or ISPA_ERR_CUDA
+ * (raw code 3: an attention CTA found its shared-memory window off a 1 KB
+ * boundary and wrote nothing).  Synchronises the device with a blocking copy
+ * of one word.  *code (nullable, host) gets the raw code. */
 ISPA_API ispa_status ispa_last_device_error(int32_t* code);
 
 /* Bound of every device-side wait, in nanoseconds (default 1e9).  Applies to
@@ -148,7 +152,7 @@ ISPA_API uint64_t ispa_set_wait_limit_ns(uint64_t ns);
 ISPA_API ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream);
 
 /* Copy (without clearing) the device error record of the current device:
- * rec8[0] = code (0 none, 1 timeout), then the first failing wait: [1] wait
+ * rec8[0] = code (0 none, 1 timeout, 3 layout), then the first failing wait: [1] wait
  * site, [2] blockIdx.x, [3] blockIdx.y, [4] threadIdx.x, [5] barrier shared
  * address, [6] parity, [7] tile index.  rec8: host array of 8 int32.
  * Synchronises like ispa_last_device_error. */

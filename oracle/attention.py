@@ -13,7 +13,7 @@ Paper basis
     scaled scores.
   * Eq. 11-12: LSE_full = log(exp(LSE_loc) + exp(LSE_hist)) and
     A_full = exp(LSE_loc - LSE_full) O_loc + exp(LSE_hist - LSE_full) O_hist.
-  * Discrepancy (Sec. 3.1 "monitors the output discrepancy"): the paper does
+  * Discrepancy (Sec. 3.1, tracked between the two branches): the paper does
     not define it; the reading used is disc_t = || A_full,t - A_loc,t ||_2
     over all D features of token t, plus the sum of disc_t^2 over tokens.
 

@@ -311,6 +311,7 @@ ispa_status ispa_last_device_error(int32_t* code) {
   if (cudaMemcpyToSymbol(g_status, zero, sizeof(zero)) != cudaSuccess) return ISPA_ERR_CUDA;
   if (code) *code = rec[0];
   if (rec[0] == DEVERR_TIMEOUT) return ISPA_ERR_TIMEOUT;
+  if (rec[0] == DEVERR_LAYOUT) return ISPA_ERR_CUDA;
   return ISPA_OK;
 }
 

@@ -17,11 +17,13 @@
 // CTA = one head x one tile of 128 queries, key tiles of 176 keys; 320 threads:
 //   warps 0-7  softmax: warp w owns query rows 32(w%4)..+31 (its TMEM lane
 //              quarter) and the score columns 88(w/4)..+87 of every key tile,
-//              so each row's 128 scores are split over two warps that swap
+//              so each row's 176 scores are split over two warps that swap
 //              their partial row maxima through shared memory once per tile;
 //   warp 8     TMA producer (Q once, then K/V tiles into staged rings);
 //   warp 9     TMEM allocator and UMMA issuer.
 // TMEM columns: S0 [0,176) S1 [176,352) O [352,352+d).
+// Shared memory (d = 128): Q 32 KB, two K and two V stages of 44 KB, 2 KB of
+// row-max exchange (reused by the epilogue), barriers: 215,184 bytes.
 // Per key tile j: S_j = Q K_j^T (SS-UMMA, M=128 N=176, fp32 in TMEM) -> softmax
 // warps read S_j, update the row max (lazy rescale of O only when the max grows
 // by more than 2^8), write P_j = exp2(.) as bf16 over the first 88 columns of
@@ -30,7 +32,8 @@
 // work on S_j; S_{j+2} overwrites P_j only after PV_j, which the in-order
 // execution of one thread's UMMAs guarantees.  176-key tiles put more work in
 // each UMMA instruction than 128 (the per-instruction cost, not the work, bounds
-// 128x128x16 UMMAs here) while S0 + S1 + O still fit the 512 TMEM columns.
+// 128x128x16 UMMAs here).  192-key tiles (S0 + S1 + O = all 512 columns) measured
+// about 1% slower: the PV chain (11 vs 12 dependent N=128 UMMAs) sets the pace.
 //
 // Every wait is bounded; after a timeout the softmax warps keep executing
 // their named barriers (without touching TMEM) so no warp is left behind.
@@ -72,10 +75,11 @@ struct Cfg {
   static constexpr int OFF_K = Q_TILE;
   static constexpr int OFF_V = OFF_K + KST * KV_TILE;
   static constexpr int OFF_X = OFF_V + VST * KV_TILE;          // exchange arrays (fp32)
-  static constexpr int X_FLOATS = 2 * 2 * BM + 2 * BM + 2 * BM;  // max[2][2][BM], l[2][BM], sq[2][BM]
+  static constexpr int X_FLOATS = 2 * 2 * BM;  // max[parity][half][BM]; the epilogue reuses it
   static constexpr int OFF_BAR = OFF_X + X_FLOATS * 4;
   static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
-  static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16 + 1024;  // + tmem slot/abort + alignment
+  static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;  // + tmem slot / abort flag / spare
+  static_assert(SMEM <= 232448, "shared memory per CTA");
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
   static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
@@ -144,13 +148,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_kc,
                 const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
   using C = Cfg<HD>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  // The dynamic shared window must start on a 1 KB boundary (the swizzle atoms of the
+  // TMA boxes); the declaration asks for it and the check below enforces it.
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
   const uint32_t sbase = smem_u32(smem);
+  if (sbase & 1023u) {  // uniform over the CTA; nothing is initialised yet
+    if (threadIdx.x == 0) record_error(p.status, DEVERR_LAYOUT, 0, sbase, 0, 0);
+    return;
+  }
   float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [parity][half][row]
-  float* x_l = x_max + 4 * BM;                                // [half][row]
-  float* x_sq = x_l + 2 * BM;                                 // [half][row]
   uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -338,7 +345,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // Normalise O by the full-row l and store this warp's half of the row (bf16); optional
     // LSE; optional discrepancy partial sum_d (A_full - A_loc)^2 of this head on the stored
     // bf16 values.  Executes the same two named barriers whether or not `live`.
-    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc) {
+    // xb = parity of the next key tile: the max-exchange block of that parity is idle (its
+    // last readers passed the previous tile's barrier) and holds the l exchange; the other
+    // block, still read by the partner warp until the first barrier below, then holds sq.
+    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc, int xb) {
+      float* x_l = x_max + (xb * 2) * BM;          // [half][row]
+      float* x_sq = x_max + ((xb ^ 1) * 2) * BM;   // [half][row]
       x_l[half * BM + row] = l_run;
       soft_barrier();
       const float l_row = l_run + x_l[(half ^ 1) * BM + row];
@@ -391,7 +403,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
         if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 7, j));
         if (ok) tc_fence_after();
-        emit(ok, p.out_loc, p.lse_loc, false);
+        emit(ok, p.out_loc, p.lse_loc, false, j & 1);
       }
       if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
       if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 0);
@@ -486,8 +498,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int jl = n_tiles - 1;
       if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc, 11, jl));
       if (ok) tc_fence_after();
-      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
-      emit(ok, p.out, p.lse, p.dual != 0);
+      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false, n_tiles & 1);
+      emit(ok, p.out, p.lse, p.dual != 0, n_tiles & 1);
     }
   }
 

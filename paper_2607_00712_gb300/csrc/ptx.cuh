@@ -14,7 +14,8 @@
 namespace ispa {
 
 // Device status codes (written into the library status word).
-enum : int { DEVERR_NONE = 0, DEVERR_TIMEOUT = 1, DEVERR_NOT_SPD = 2 };
+// DEVERR_LAYOUT: a kernel found its shared-memory window misaligned and did no work.
+enum : int { DEVERR_NONE = 0, DEVERR_TIMEOUT = 1, DEVERR_NOT_SPD = 2, DEVERR_LAYOUT = 3 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

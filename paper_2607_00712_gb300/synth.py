@@ -5,7 +5,7 @@ none of ISPA's arithmetic (no attention, no least squares, no ring mapping).
 Both the CUDA path and the fp64 oracle consume exactly the arrays made here.
 
 Input recipe (stand-in for the post-RoPE activations of an autoregressive
-video DiT, Sec. 2 "KV injection", Eq. 3):
+video DiT, Sec. 2, the KV injection of Eq. 3):
   * q, k, v ~ N(0, 1), drawn in fp32 with numpy's PCG64: each array gets its
     own child of SeedSequence(seed), split into 2^20-value chunks with one
     grandchild stream each (drawn in parallel threads, so the values depend
