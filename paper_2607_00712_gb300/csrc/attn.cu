@@ -11,9 +11,11 @@
 //     materialised, every key is visited once, and the fusion costs one
 //     extra read of O from TMEM per row.
 //
-// Tensor maps: the ring as (d, cap*P, H) and the chunk tensors q/k_cur/v_cur
-// as (d, H, n_q), boxes of 64 x 128 rows x 1 head with 128-byte swizzle, which
-// is the K-major (Q, K) and MN-major (V) UMMA operand layout.
+// Tensor maps: every operand as (64 columns, rows, d/64 column blocks, heads), the
+// ring with rows = cap*P slots and the chunk tensors q/k_cur/v_cur with rows = n_q;
+// one box (64, tile rows, d/64, 1) with 128-byte swizzle fetches a whole Q, K or V
+// tile in one request as d/64 consecutive [rows][128 B] blocks, which is the
+// K-major (Q, K) and MN-major (V) UMMA operand layout.
 // CTA = one head x one tile of 128 queries, key tiles of 176 keys; 320 threads:
 //   warps 0-7  softmax: warp w owns query rows 32(w%4)..+31 (its TMEM lane
 //              quarter) and the score columns 88(w/4)..+87 of every key tile,
@@ -226,8 +228,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (lane == 0) {
       const uint32_t sQ = sbase + C::OFF_Q;
       mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
-#pragma unroll
-      for (int x = 0; x < C::NBOX; ++x) tma_load_3d(sQ + x * C::QBOX, &tm_q, b.q_full, 64 * x, head, q0);
+      tma_load_4d(sQ, &tm_q, b.q_full, 0, q0, 0, head);
       // Loads are issued in the order their stages free up: the UMMA stream is
       // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so stages free as K_t (after S_{t-KST}) then
       // V_{t-1} (after PV_{t-1-VST}); V therefore trails K by one tile.
@@ -241,11 +242,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (!mbar_wait(b.k_empty0 + 8 * ks, ((t / C::KST) & 1) ^ 1, wc, 1, t)) break;
           mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::KV_TILE);
           const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
-#pragma unroll
-          for (int x = 0; x < C::NBOX; ++x) {
-            if (chunk) tma_load_3d(sK + x * C::KBOX, &tm_kc, b.k_full0 + 8 * ks, 64 * x, head, row);
-            else tma_load_3d(sK + x * C::KBOX, &tm_kr, b.k_full0 + 8 * ks, 64 * x, row, head);
-          }
+          tma_load_4d(sK, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0, row, 0, head);
           nk = t + 1;
           trace_event(p.trace, p.trace_tiles, t, 6);
           next_tile(p, kseg, koff);
@@ -258,11 +255,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
           mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::KV_TILE);
           const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
-#pragma unroll
-          for (int x = 0; x < C::NBOX; ++x) {
-            if (chunk) tma_load_3d(sV + x * C::KBOX, &tm_vc, b.v_full0 + 8 * vs, 64 * x, head, row);
-            else tma_load_3d(sV + x * C::KBOX, &tm_vr, b.v_full0 + 8 * vs, 64 * x, row, head);
-          }
+          tma_load_4d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0, row, 0, head);
           nv = j + 1;
           trace_event(p.trace, p.trace_tiles, j, 7);
           next_tile(p, vseg, voff);

@@ -10,9 +10,15 @@
 //   G tile: a^T a;   X tile: a^T hi + a^T lo;   S tile: hi^T hi + hi^T lo + lo^T hi
 // (the lo^T lo term is below fp32 resolution and dropped).  Both operands
 // are token-major [T][D] in HBM, i.e. MN-major for the UMMA, staged by TMA in
-// 64-token x 64-feature boxes with 128-byte swizzle.  Tokens are split across
-// CTAs (blockIdx.y) and each CTA adds its partial tile into the fp32 state
-// with vector atomics.
+// 64-token x 64-feature boxes with 128-byte swizzle.
+//
+// Work split (stream-K): the tiles are laid end to end as one sequence of
+// steps (tile, pass, 64-token block) -- G tiles (1 pass each), X tiles (2),
+// S tiles (3) -- and a persistent grid of one CTA per SM takes equal
+// contiguous ranges of it.  A CTA's range covers the tail of one tile, some
+// whole tiles and the head of another; each such segment is summed in one of
+// two TMEM accumulators and added into the fp32 state with vector atomics by
+// the epilogue warps while the UMMA warp already fills the other accumulator.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -37,9 +43,12 @@ struct GCfg {
   static constexpr int B_BYTES = (BN / 64) * BOX;
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int OFF_BAR = GST * STAGE;
-  static constexpr int SMEM = OFF_BAR + (2 * GST + 2) * 8 + 16 + 1024;
+  static constexpr int N_BAR = 2 * GST + 2 + 2 + 1;   // full/empty stages, acc full/empty x2, drain
+  static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
+  static_assert(STAGE % 1024 == 0 && BOX % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
   static constexpr uint32_t IDESC = idesc_bf16(GM, BN, true, true);
-  static constexpr uint32_t TMEM_COLS = BN;  // 128 or 256, both powers of two
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators: 256 or 512 columns
 };
 
 // Operand sources of the passes of each block type: 0 = A_loc, 1 = hi, 2 = lo.
@@ -57,12 +66,35 @@ struct GramParams {
   int32_t D;
   int32_t T;
   int32_t n_ktiles;   // ceil(T / GK)
-  int32_t kt_per_split;
+  int32_t n_upper;    // upper-block tiles of G (and of S)
+  int32_t n_full;     // tiles of X
+  int32_t total;      // steps over all tiles
   float* gram;        // [2D][2D]
   int* status;
   uint64_t wait_limit_ns;
   uint32_t* heartbeat;
 };
+
+// Step g of the global sequence -> tile (item, numbered as decode_tile expects) and its
+// first step.  Tiles: n_upper G tiles of n_kt steps, n_full X tiles of 2 n_kt, n_upper S
+// tiles of 3 n_kt.
+__device__ __forceinline__ void step_item(const GramParams& p, int g, int& item, int& first) {
+  const int n_kt = p.n_ktiles;
+  const int g_end = p.n_upper * n_kt;
+  const int x_end = g_end + p.n_full * 2 * n_kt;
+  if (g < g_end) {
+    item = g / n_kt;
+    first = item * n_kt;
+  } else if (g < x_end) {
+    const int i = (g - g_end) / (2 * n_kt);
+    item = p.n_upper + i;
+    first = g_end + i * 2 * n_kt;
+  } else {
+    const int i = (g - x_end) / (3 * n_kt);
+    item = p.n_upper + p.n_full + i;
+    first = x_end + i * 3 * n_kt;
+  }
+}
 
 // Decode blockIdx.x into (kind, row block, col block).  Items: upper G tiles,
 // then all X tiles, then upper S tiles.
@@ -127,34 +159,34 @@ __global__ void __launch_bounds__(G_THREADS, 1)
     gram_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_hi,
                 const __grid_constant__ CUtensorMap tm_lo, const GramParams p) {
   using C = GCfg<BN>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
   const uint32_t sbase = smem_u32(smem);
+  if (sbase & 1023u) {  // uniform over the CTA; nothing is initialised yet
+    if (threadIdx.x == 0) record_error(p.status, DEVERR_LAYOUT, 0, sbase, 0, 1);
+    return;
+  }
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * GST + 2);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::N_BAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * GST, acc_bar = empty0 + 8 * GST,
-                 drain_bar = acc_bar + 8;
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * GST, accf0 = empty0 + 8 * GST,
+                 acce0 = accf0 + 16, drain_bar = acce0 + 16;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int kind, bi, bj;
-  decode_tile<BN>(blockIdx.x, p.D, kind, bi, bj);
-  const int kt0 = blockIdx.y * p.kt_per_split;
-  const int kt1 = min(p.n_ktiles, kt0 + p.kt_per_split);
-  const int n_kt = kt1 - kt0;
-  const int n_pass = kNumPasses[kind];
-  const int total_steps = n_pass * n_kt;
-  // feature offsets inside the [T][D] operands
-  const int fa = bi * GM;   // rows of the output tile = features of operand A
-  const int fb = bj * BN;   // cols of the output tile = features of operand B
+  // this CTA's contiguous step range
+  const int g0 = static_cast<int>(static_cast<int64_t>(p.total) * blockIdx.x / gridDim.x);
+  const int g1 = static_cast<int>(static_cast<int64_t>(p.total) * (blockIdx.x + 1) / gridDim.x);
+  const int n_kt = p.n_ktiles;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < GST; ++i) {
       mbar_init(full0 + 8 * i, 1);
       mbar_init(empty0 + 8 * i, 1);
     }
-    mbar_init(acc_bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(accf0 + 8 * i, 1);
+      mbar_init(acce0 + 8 * i, 128);
+    }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -172,66 +204,101 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
 
   if (warp == 0) {
-    if (lane == 0 && total_steps > 0) {
-      const CUtensorMap* maps[3] = {&tm_a, &tm_hi, &tm_lo};
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && g1 > g0) {
+      auto map_of = [&](int w) { return w == 0 ? &tm_a : (w == 1 ? &tm_hi : &tm_lo); };
       int issued = 0;
-      for (int s = 0; s < total_steps; ++s) {
-        const int pass = s / n_kt;
-        const int tok = (kt0 + s % n_kt) * GK;
-        const int st = s % GST;
-        if (!mbar_wait(empty0 + 8 * st, ((s / GST) & 1) ^ 1, wc, 21, s)) break;
+      int item = -1, first = 0, kind = 0, bi = 0, bj = 0;
+      for (int g = g0; g < g1; ++g) {
+        const int i = g - g0;
+        if (item < 0 || g >= first + kNumPasses[kind] * n_kt) {
+          step_item(p, g, item, first);
+          decode_tile<BN>(item, p.D, kind, bi, bj);
+        }
+        const int local = g - first;
+        const int pass = local / n_kt;
+        const int tok = (local % n_kt) * GK;
+        const int st = i % GST;
+        if (!mbar_wait(empty0 + 8 * st, ((i / GST) & 1) ^ 1, wc, 21, i)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
         const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
-        const CUtensorMap* ma = maps[kPasses[kind][pass].a];
-        const CUtensorMap* mb = maps[kPasses[kind][pass].b];
+        const CUtensorMap* ma = map_of(kPasses[kind][pass].a);
+        const CUtensorMap* mb = map_of(kPasses[kind][pass].b);
 #pragma unroll
-        for (int x = 0; x < GM / 64; ++x) tma_load_2d(sa + x * C::BOX, ma, full0 + 8 * st, fa + 64 * x, tok);
+        for (int x = 0; x < GM / 64; ++x) tma_load_2d(sa + x * C::BOX, ma, full0 + 8 * st, bi * GM + 64 * x, tok);
 #pragma unroll
-        for (int x = 0; x < BN / 64; ++x) tma_load_2d(sb + x * C::BOX, mb, full0 + 8 * st, fb + 64 * x, tok);
-        issued = s + 1;
+        for (int x = 0; x < BN / 64; ++x) tma_load_2d(sb + x * C::BOX, mb, full0 + 8 * st, bj * BN + 64 * x, tok);
+        issued = i + 1;
       }
-      for (int s = issued > GST ? issued - GST : 0; s < issued; ++s)
-        mbar_wait_drain(full0 + 8 * (s % GST), (s / GST) & 1, G_DRAIN_NS);
+      for (int i = issued > GST ? issued - GST : 0; i < issued; ++i)
+        mbar_wait_drain(full0 + 8 * (i % GST), (i / GST) & 1, G_DRAIN_NS);
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0 && total_steps > 0) {
+    // ------------------------------------------------------------ UMMA issuer
+    if (lane == 0 && g1 > g0) {
       bool ok = true;
-      for (int s = 0; s < total_steps; ++s) {
-        const int st = s % GST;
-        if (!mbar_wait(full0 + 8 * st, (s / GST) & 1, wc, 22, s)) {
+      int seg = 0, item = -1, first = 0, last = 0;
+      for (int g = g0; ok && g < g1; ++g) {
+        const int i = g - g0;
+        if (g == g0 || g >= last) {   // a new segment starts: claim accumulator seg & 1
+          if (g > g0) ++seg;
+          step_item(p, g, item, first);
+          int kind, bi, bj;
+          decode_tile<BN>(item, p.D, kind, bi, bj);
+          last = first + kNumPasses[kind] * n_kt;
+          const int b = seg & 1;
+          if (!mbar_wait(acce0 + 8 * b, ((seg >> 1) & 1) ^ 1, wc, 24, seg)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+        }
+        const int st = i % GST;
+        if (!mbar_wait(full0 + 8 * st, (i / GST) & 1, wc, 22, i)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
+        const uint32_t acc = tmem + (seg & 1) * BN;
+        const bool seg_first = (g == g0) || (g == first);
 #pragma unroll
         for (int k = 0; k < GK / 16; ++k)
-          umma_ss(tmem, sw128_desc(sa + k * 2048, C::BOX, 1024), sw128_desc(sb + k * 2048, C::BOX, 1024),
-                  C::IDESC, (s > 0 || k > 0) ? 1u : 0u);
+          umma_ss(acc, sw128_desc(sa + k * 2048, C::BOX, 1024), sw128_desc(sb + k * 2048, C::BOX, 1024), C::IDESC,
+                  (!seg_first || k > 0) ? 1u : 0u);
         tc_commit(empty0 + 8 * st);
+        if (g + 1 == g1 || g + 1 == last) tc_commit(accf0 + 8 * (seg & 1));
       }
-      if (ok) tc_commit(acc_bar);
       tc_commit(drain_bar);
       mbar_wait_drain(drain_bar, 0, G_DRAIN_NS);
     }
     __syncwarp();
-  } else if (total_steps > 0) {
-    // epilogue: warp w reads TMEM lanes 32*(w%4) .. +31 = output rows
+  } else if (g1 > g0) {
+    // ------------------------------------------------------------ epilogue (warps 2-5)
+    // warp w reads TMEM lanes 32*(w%4) .. +31 = output rows of the tile
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, wc, 23, 0));
-    if (ok) {
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    int item_a, first_a, item_b, first_b;
+    step_item(p, g0, item_a, first_a);
+    step_item(p, g1 - 1, item_b, first_b);
+    bool ok = true;
+    for (int seg = 0; seg <= item_b - item_a; ++seg) {
+      const int b = seg & 1;
+      ok = ok && __all_sync(0xffffffffu, mbar_wait(accf0 + 8 * b, (seg >> 1) & 1, wc, 23, seg));
+      if (!ok) break;
       tc_fence_after();
+      int kind, bi, bj;
+      decode_tile<BN>(item_a + seg, p.D, kind, bi, bj);
       const int D = p.D;
-      const int row0 = (kind == 2 ? D : 0) + fa;
-      const int col0 = (kind == 0 ? 0 : D) + fb;
+      const int row0 = (kind == 2 ? D : 0) + bi * GM;
+      const int col0 = (kind == 0 ? 0 : D) + bj * BN;
       float* grow = p.gram + static_cast<size_t>(row0 + r) * (2 * D) + col0;
-      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         uint32_t v[32];
-        tmem_ld32(taddr + 32 * c, v);
+        tmem_ld32(lane_base + b * BN + 32 * c, v);
         tmem_wait_ld32(v);
         float4* g4 = reinterpret_cast<float4*>(grow + 32 * c);
 #pragma unroll
@@ -239,6 +306,8 @@ __global__ void __launch_bounds__(G_THREADS, 1)
           atomicAdd(g4 + q, make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
                                         __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3])));
       }
+      tc_fence_before();
+      mbar_arrive(acce0 + 8 * b);   // accumulator b may be overwritten
     }
   }
 
@@ -278,21 +347,22 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   const int RB = D / GM, CB = D / BN;
   int n_upper = 0;
   for (int r = 0; r < RB; ++r) n_upper += CB - (r * GM) / BN;
-  const int n_items = 2 * n_upper + RB * CB;
   GramParams p;
   p.D = D;
   p.T = static_cast<int32_t>(T);
   p.n_ktiles = static_cast<int32_t>((T + GK - 1) / GK);
-  // token splits: aim at >= 3 CTAs per SM over all items, at least 8 token tiles each
-  int splits = (3 * sms + n_items - 1) / n_items;
-  splits = max(1, min(splits, p.n_ktiles / 8 > 0 ? p.n_ktiles / 8 : 1));
-  p.kt_per_split = (p.n_ktiles + splits - 1) / splits;
-  splits = (p.n_ktiles + p.kt_per_split - 1) / p.kt_per_split;
+  p.n_upper = n_upper;
+  p.n_full = RB * CB;
+  const int64_t total = static_cast<int64_t>(p.n_ktiles) * (n_upper * 1 + p.n_full * 2 + n_upper * 3);
+  if (total > INT32_MAX) return cudaErrorInvalidValue;
+  p.total = static_cast<int32_t>(total);
   p.gram = gram;
   p.status = status;
   p.wait_limit_ns = wait_limit_ns;
   p.heartbeat = hb;
-  dim3 grid(n_items, splits);
+  // one CTA per SM, each with at least 16 steps (a 1024-token run of one tile)
+  const int64_t want = (total + 15) / 16;
+  const dim3 grid(static_cast<unsigned>(want < sms ? (want > 0 ? want : 1) : sms));
   gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(ta, th, tl, p);
   return cudaGetLastError();
 }

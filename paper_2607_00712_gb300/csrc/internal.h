@@ -96,6 +96,9 @@ int* device_status_ptr();  // library status word on the current device (nullptr
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                     uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                     uint32_t b2);
+// bf16, 128-byte swizzle, rank 4 (dims / strides in bytes for dims 1-3 / box).
+bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], const uint64_t strides3[3],
+                    const uint32_t box4[4]);
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();
