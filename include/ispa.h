@@ -211,6 +211,15 @@ ISPA_API ispa_status ispa_kv_append_layers(ispa_kv_ring* rings, int32_t n_layers
 
 /* ------------------------------------------------------------ attention */
 
+/* Option bits of the *_ex attention entry points. */
+#define ISPA_ATTN_FRAME_CAUSAL 1u
+/*   ISPA_ATTN_FRAME_CAUSAL: block-causal at frame granularity inside the chunk.
+ *   Eq. 3 leaves the chunk dense (every chunk query sees every chunk key); with
+ *   this bit a query of the chunk's frame a (rows a*P .. a*P+P-1) sees the
+ *   chunk's frames 0..a only.  Past frames stay fully visible.  n_q must be a
+ *   multiple of tokens_per_frame (else ISPA_ERR_INVALID_ARG).  Unknown bits are
+ *   ISPA_ERR_INVALID_ARG.  flags = 0 is the plain entry point. */
+
 /*
  * F-layer chunk attention (Eq. 3): Q = Q_cur, K = [K_past; K_cur],
  * V = [V_past; V_cur], with K_past/V_past every resident frame of the ring.
@@ -224,6 +233,10 @@ ISPA_API ispa_status ispa_kv_append_layers(ispa_kv_ring* rings, int32_t n_layers
 ISPA_API ispa_status ispa_attn_full(const ispa_kv_ring* ring, const void* q, const void* k_cur,
                            const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
                            ispa_stream stream);
+/* ispa_attn_full with option bits (ISPA_ATTN_FRAME_CAUSAL). */
+ISPA_API ispa_status ispa_attn_full_ex(const ispa_kv_ring* ring, const void* q, const void* k_cur,
+                              const void* v_cur, int32_t n_q, float scale, uint32_t flags, void* out,
+                              float* lse, ispa_stream stream);
 
 /*
  * L-layer chunk attention (Sec. 3.3, Eq. 7): the same over the local set
@@ -234,6 +247,10 @@ ISPA_API ispa_status ispa_attn_full(const ispa_kv_ring* ring, const void* q, con
 ISPA_API ispa_status ispa_attn_local(const ispa_kv_ring* ring, ispa_window win, const void* q,
                             const void* k_cur, const void* v_cur, int32_t n_q, float scale,
                             void* out, float* lse, ispa_stream stream);
+/* ispa_attn_local with option bits (ISPA_ATTN_FRAME_CAUSAL). */
+ISPA_API ispa_status ispa_attn_local_ex(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                               const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                               uint32_t flags, void* out, float* lse, ispa_stream stream);
 
 /* Workspace bytes of ispa_attn_dual (fp32 [num_heads][n_q] partial sums). */
 ISPA_API size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q);
@@ -246,7 +263,7 @@ ISPA_API size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q);
  *   a_full, a_loc  : bf16 [n_q][num_heads * head_dim]
  *   disc           : fp32 [n_q], disc_t = || A_full,t - A_loc,t ||_2 over all
  *                    num_heads*head_dim features, taken on the stored bf16
- *                    outputs (the paper's "output discrepancy", read as this norm)
+ *                    outputs (Sec. 3.1 leaves the discrepancy undefined; read as this norm)
  *   disc_sq_sum    : fp32 device scalar, += sum_t disc_t^2 (not reset)
  *   lse_full, lse_loc : fp32 [num_heads][n_q] or NULL
  *   workspace      : >= ispa_attn_dual_workspace_size bytes
@@ -257,6 +274,13 @@ ISPA_API ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, c
                            void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
                            float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
                            ispa_stream stream);
+/* ispa_attn_dual with option bits (ISPA_ATTN_FRAME_CAUSAL: the chunk part of both
+ * A_loc and A_full is frame-causal). */
+ISPA_API ispa_status ispa_attn_dual_ex(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                              const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                              uint32_t flags, void* a_full, void* a_loc, float* disc,
+                              float* disc_sq_sum, float* lse_full, float* lse_loc, void* workspace,
+                              size_t ws_bytes, ispa_stream stream);
 
 /* Largest num_heads * n_q that ispa_attn_dual_static accepts (4 MiB of fp32). */
 #define ISPA_DUAL_STATIC_MAX_PARTIALS (1u << 20)

@@ -17,6 +17,10 @@ Paper basis
     not define it; the reading used is disc_t = || A_full,t - A_loc,t ||_2
     over all D features of token t, plus the sum of disc_t^2 over tokens.
 
+Frame-causal option (a variant beyond Eq. 3, which keeps the chunk dense): with
+frame_causal=True a query of the chunk's frame a (rows a*P .. a*P+P-1) sees the
+chunk's frames 0..a only; past frames stay fully visible.
+
 Softmax scale: the paper does not state it; 1/sqrt(d) is used when scale is 0.
 Each attention row is computed by materialising the whole score row and
 taking two passes over it (max, then exponentials); there is no tiling and no
@@ -87,23 +91,49 @@ def _rows(x, rows):
     return x if rows is None else x[rows]
 
 
-def attn_full(q, k_hist, v_hist, k_cur, v_cur, P: int, scale: float = 0.0, rows=None):
+def _attend_with_chunk(q, k_past, v_past, k_cur, v_cur, P: int, scale: float, rows, frame_causal: bool):
+    """Queries against the given past keys plus the chunk, dense or frame-causal."""
+    if not frame_causal:
+        K = np.concatenate([k_past, k_cur], axis=0)
+        V = np.concatenate([v_past, v_cur], axis=0)
+        return attend_heads(_rows(q, rows), K, V, scale)
+    n = k_cur.shape[0]
+    if n % P:
+        raise ValueError("frame-causal attention needs whole chunk frames")
+    idx = np.arange(q.shape[0]) if rows is None else np.asarray(rows)
+    H, d = q.shape[1], v_cur.shape[2]
+    out = np.zeros((len(idx), H, d))
+    lse = np.zeros((H, len(idx)))
+    for a in range(n // P):                   # queries of chunk frame a
+        sel = np.nonzero(idx // P == a)[0]
+        if len(sel) == 0:
+            continue
+        K = np.concatenate([k_past, k_cur[:(a + 1) * P]], axis=0)
+        V = np.concatenate([v_past, v_cur[:(a + 1) * P]], axis=0)
+        out[sel], lse[:, sel] = attend_heads(q[idx[sel]], K, V, scale)
+    return out, lse
+
+
+def attn_full(q, k_hist, v_hist, k_cur, v_cur, P: int, scale: float = 0.0, rows=None,
+              frame_causal: bool = False):
     """F-layer step: every past frame plus the chunk (Eq. 3).
 
     rows: optional query-row indices (rows are independent, so a subset is
     exact for those rows).  Returns (out [n, H, d], lse [H, n]).
     """
     F = k_hist.shape[0] // P
-    K, V = key_set(k_hist, v_hist, k_cur, v_cur, list(range(F)), P)
-    return attend_heads(_rows(q, rows), K, V, default_scale(q.shape[2], scale))
+    frames = list(range(F))
+    return _attend_with_chunk(q, gather_frames(k_hist, frames, P), gather_frames(v_hist, frames, P), k_cur,
+                              v_cur, P, default_scale(q.shape[2], scale), rows, frame_causal)
 
 
 def attn_local(q, k_hist, v_hist, k_cur, v_cur, P: int, n_sink: int, n_recent: int,
-               scale: float = 0.0, rows=None):
+               scale: float = 0.0, rows=None, frame_causal: bool = False):
     """L-layer step: sink frames, the n_recent newest past frames, the chunk (Eq. 7)."""
     F = k_hist.shape[0] // P
-    K, V = key_set(k_hist, v_hist, k_cur, v_cur, local_past_frames(F, n_sink, n_recent), P)
-    return attend_heads(_rows(q, rows), K, V, default_scale(q.shape[2], scale))
+    frames = local_past_frames(F, n_sink, n_recent)
+    return _attend_with_chunk(q, gather_frames(k_hist, frames, P), gather_frames(v_hist, frames, P), k_cur,
+                              v_cur, P, default_scale(q.shape[2], scale), rows, frame_causal)
 
 
 def attn_hist(q, k_hist, v_hist, P: int, n_sink: int, n_recent: int, scale: float = 0.0,
@@ -127,7 +157,7 @@ def discrepancy(a_full: np.ndarray, a_loc: np.ndarray):
 
 
 def attn_dual(q, k_hist, v_hist, k_cur, v_cur, P: int, n_sink: int, n_recent: int,
-              scale: float = 0.0, rows=None):
+              scale: float = 0.0, rows=None, frame_causal: bool = False):
     """Warmup dual step: A_full and A_loc of the same queries (Sec. 3.1, 3.4).
 
     A_full is computed directly over the full set (not through the fusion of
@@ -135,8 +165,9 @@ def attn_dual(q, k_hist, v_hist, k_cur, v_cur, P: int, n_sink: int, n_recent: in
     Returns dict with a_full, a_loc [n, H, d], lse_full, lse_loc [H, n],
     disc [n], disc_sq_sum.
     """
-    a_full, lse_full = attn_full(q, k_hist, v_hist, k_cur, v_cur, P, scale, rows)
-    a_loc, lse_loc = attn_local(q, k_hist, v_hist, k_cur, v_cur, P, n_sink, n_recent, scale, rows)
+    a_full, lse_full = attn_full(q, k_hist, v_hist, k_cur, v_cur, P, scale, rows, frame_causal)
+    a_loc, lse_loc = attn_local(q, k_hist, v_hist, k_cur, v_cur, P, n_sink, n_recent, scale, rows,
+                                frame_causal)
     disc, disc_sq_sum = discrepancy(a_full, a_loc)
     return dict(a_full=a_full, a_loc=a_loc, lse_full=lse_full, lse_loc=lse_loc,
                 disc=disc, disc_sq_sum=disc_sq_sum)

@@ -10,7 +10,8 @@ from __future__ import annotations
 
 import ctypes
 import os
-from ctypes import POINTER, Structure, c_char_p, c_double, c_float, c_int32, c_int64, c_size_t, c_uint64, c_void_p
+from ctypes import (POINTER, Structure, c_char_p, c_double, c_float, c_int32, c_int64, c_size_t, c_uint32, c_uint64,
+                    c_void_p)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libispa.so")
@@ -23,6 +24,7 @@ ISPA_ERR_NOT_SPD = 4
 ISPA_ERR_TIMEOUT = 5
 ISPA_ERR_CUDA = 6
 ISPA_ERR_WORKSPACE = 7
+ISPA_ATTN_FRAME_CAUSAL = 1   # option bit of the *_ex attention entry points
 MAX_RANGES = 4
 
 
@@ -82,6 +84,13 @@ _SIGS = {
                                  c_void_p, c_void_p]),
     "ispa_attn_local": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                   c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_full_ex": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_int32, c_float, c_uint32,
+                                    c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_local_ex": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
+                                     c_uint32, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_dual_ex": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
+                                    c_uint32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                    c_void_p, c_size_t, c_void_p]),
     "ispa_attn_dual_workspace_size": (c_size_t, [c_int32, c_int32]),
     "ispa_attn_dual": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                  c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -212,6 +221,27 @@ def ispa_attn_local(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale:
                     stream=None) -> None:
     _check(lib().ispa_attn_local(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
                                  _ptr(out), _ptr(lse), _stream(stream)), "ispa_attn_local")
+
+
+def ispa_attn_full_ex(ring: KVRing, q, k_cur, v_cur, n_q: int, scale: float, flags: int, out, lse=None,
+                      stream=None) -> None:
+    _check(lib().ispa_attn_full_ex(ctypes.byref(ring), _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale, flags,
+                                   _ptr(out), _ptr(lse), _stream(stream)), "ispa_attn_full_ex")
+
+
+def ispa_attn_local_ex(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, flags: int, out,
+                       lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_local_ex(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
+                                    flags, _ptr(out), _ptr(lse), _stream(stream)), "ispa_attn_local_ex")
+
+
+def ispa_attn_dual_ex(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, flags: int, a_full,
+                      a_loc, disc, disc_sq_sum, lse_full=None, lse_loc=None, workspace=None, ws_bytes: int = 0,
+                      stream=None) -> None:
+    _check(lib().ispa_attn_dual_ex(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
+                                   flags, _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum),
+                                   _ptr(lse_full), _ptr(lse_loc), _ptr(workspace), ws_bytes, _stream(stream)),
+           "ispa_attn_dual_ex")
 
 
 def ispa_attn_dual_workspace_size(num_heads: int, n_q: int) -> int:

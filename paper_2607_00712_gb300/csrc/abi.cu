@@ -209,11 +209,13 @@ int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
 }
 
 ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, const void* q,
-                        const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                        const void* k_cur, const void* v_cur, int32_t n_q, float scale, uint32_t flags,
                         void* out, void* out_loc, float* lse, float* lse_loc, float* disc_part,
                         cudaStream_t stream) {
   ispa_status st = check_ring(ring);
   if (st != ISPA_OK) return st;
+  if (flags & ~static_cast<uint32_t>(ISPA_ATTN_FRAME_CAUSAL)) return ISPA_ERR_INVALID_ARG;
+  if ((flags & ISPA_ATTN_FRAME_CAUSAL) && n_q % ring->tokens_per_frame != 0) return ISPA_ERR_INVALID_ARG;
   if (n_q <= 0 || !aligned16(q) || !aligned16(k_cur) || !aligned16(v_cur) || !aligned16(out) ||
       !aligned16(ring->k) || !aligned16(ring->v))
     return ISPA_ERR_INVALID_ARG;
@@ -255,6 +257,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
     p.n_tiles = tiles;
   }
   p.dual = mode == MODE_DUAL ? 1 : 0;
+  p.causal_p = (flags & ISPA_ATTN_FRAME_CAUSAL) ? P : 0;
   const float sc = scale == 0.f ? 1.f / sqrtf(static_cast<float>(HD)) : scale;
   p.scale_log2 = sc * 1.4426950408889634f;
   p.wait_limit_ns = g_wait_limit;
@@ -439,25 +442,37 @@ ispa_status ispa_kv_append(ispa_kv_ring* ring, const void* k_new, const void* v_
   return ispa_kv_append_layers(ring, 1, k, v, n_frames, stream);
 }
 
+ispa_status ispa_attn_full_ex(const ispa_kv_ring* ring, const void* q, const void* k_cur,
+                              const void* v_cur, int32_t n_q, float scale, uint32_t flags, void* out,
+                              float* lse, ispa_stream stream) {
+  return attn_common(MODE_FULL, ring, ispa_window{0, 0}, q, k_cur, v_cur, n_q, scale, flags, out, nullptr,
+                     lse, nullptr, nullptr, stream);
+}
+
 ispa_status ispa_attn_full(const ispa_kv_ring* ring, const void* q, const void* k_cur,
                            const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
                            ispa_stream stream) {
-  return attn_common(MODE_FULL, ring, ispa_window{0, 0}, q, k_cur, v_cur, n_q, scale, out, nullptr,
-                     lse, nullptr, nullptr, stream);
+  return ispa_attn_full_ex(ring, q, k_cur, v_cur, n_q, scale, 0u, out, lse, stream);
+}
+
+ispa_status ispa_attn_local_ex(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                               const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                               uint32_t flags, void* out, float* lse, ispa_stream stream) {
+  return attn_common(MODE_LOCAL, ring, win, q, k_cur, v_cur, n_q, scale, flags, out, nullptr, lse, nullptr,
+                     nullptr, stream);
 }
 
 ispa_status ispa_attn_local(const ispa_kv_ring* ring, ispa_window win, const void* q,
                             const void* k_cur, const void* v_cur, int32_t n_q, float scale,
                             void* out, float* lse, ispa_stream stream) {
-  return attn_common(MODE_LOCAL, ring, win, q, k_cur, v_cur, n_q, scale, out, nullptr, lse, nullptr,
-                     nullptr, stream);
+  return ispa_attn_local_ex(ring, win, q, k_cur, v_cur, n_q, scale, 0u, out, lse, stream);
 }
 
 ispa_status ispa_attn_hist(const ispa_kv_ring* ring, ispa_window win, const void* q, int32_t n_q, float scale,
                            void* out, float* lse, ispa_stream stream) {
   if (!lse) return ISPA_ERR_INVALID_ARG;
   // the chunk tensors are not read in this mode; q stands in for them in the unused maps
-  return attn_common(MODE_HIST, ring, win, q, q, q, n_q, scale, out, nullptr, lse, nullptr, nullptr, stream);
+  return attn_common(MODE_HIST, ring, win, q, q, q, n_q, scale, 0u, out, nullptr, lse, nullptr, nullptr, stream);
 }
 
 size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q) {
@@ -465,22 +480,31 @@ size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q) {
   return static_cast<size_t>(num_heads) * n_q * sizeof(float);
 }
 
-ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void* q,
-                           const void* k_cur, const void* v_cur, int32_t n_q, float scale,
-                           void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
-                           float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
-                           ispa_stream stream) {
+ispa_status ispa_attn_dual_ex(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                              const void* k_cur, const void* v_cur, int32_t n_q, float scale, uint32_t flags,
+                              void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                              float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                              ispa_stream stream) {
   if (!ring || !disc || !disc_sq_sum) return ISPA_ERR_INVALID_ARG;
   const size_t need = ispa_attn_dual_workspace_size(ring->num_heads, n_q);
   if (need == 0) return ISPA_ERR_INVALID_ARG;
   if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
   float* part = static_cast<float*>(workspace);
-  const ispa_status st = attn_common(MODE_DUAL, ring, win, q, k_cur, v_cur, n_q, scale, a_full,
+  const ispa_status st = attn_common(MODE_DUAL, ring, win, q, k_cur, v_cur, n_q, scale, flags, a_full,
                                      a_loc, lse_full, lse_loc, part, stream);
   if (st != ISPA_OK) return st;
   if (launch_disc_reduce(part, ring->num_heads, n_q, disc, disc_sq_sum, stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   return ISPA_OK;
+}
+
+ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void* q,
+                           const void* k_cur, const void* v_cur, int32_t n_q, float scale,
+                           void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                           float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                           ispa_stream stream) {
+  return ispa_attn_dual_ex(ring, win, q, k_cur, v_cur, n_q, scale, 0u, a_full, a_loc, disc, disc_sq_sum,
+                           lse_full, lse_loc, workspace, ws_bytes, stream);
 }
 
 size_t ispa_ls_state_bytes(int32_t dim) {

@@ -1,7 +1,8 @@
 // Chunk-step attention against the KV ring on sm_103a (tcgen05 + TMEM + TMA).
 //
 // One kernel serves the three modes of ISPA's attention:
-//   * F-layer (Eq. 3): keys = every resident past frame plus the chunk;
+//   * F-layer (Eq. 3): keys = every resident past frame plus the chunk (dense, or
+//     optionally frame-causal: a query sees the chunk's frames up to its own);
 //   * L-layer (Sec. 3.3, Eq. 7): keys = sink + recent window + chunk;
 //   * dual warmup (Sec. 3.1 phase 1, Sec. 3.4): the local segments are visited
 //     first; after the last local tile the running online-softmax state
@@ -410,7 +411,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
 #pragma unroll
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
-        const int vloc = valid - half * HALF_COLS;   // valid columns of this half
+        int vloc = valid - half * HALF_COLS;   // valid columns of this half
+        if (p.causal_p != 0 && p.seg[seg].src != 0) {
+          // frame-causal chunk: this row sees chunk keys below the end of its own frame
+          const int kc0 = p.seg[seg].start + off + half * HALF_COLS;   // chunk index of column 0
+          vloc = min(vloc, (qrow / p.causal_p + 1) * p.causal_p - kc0);
+        }
         if (vloc < HALF_COLS) {
 #pragma unroll
           for (int i = 0; i < HALF_COLS; ++i)

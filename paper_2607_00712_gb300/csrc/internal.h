@@ -33,7 +33,8 @@ struct AttnParams {
   int32_t n_local_tiles;   // dual: tiles of the local set (they come first)
   int32_t dual;            // 1 = emit A_loc snapshot and discrepancy partials
   float scale_log2;        // softmax scale * log2(e)
-  int32_t pad;
+  int32_t causal_p;        // frame-causal chunk: tokens per frame (query row r sees chunk keys
+                           // < (r / causal_p + 1) * causal_p); 0 = the chunk is dense
   uint64_t wait_limit_ns;  // bounded-wait limit
   AttnSeg seg[kMaxSegs];
   __nv_bfloat16* out;      // [n_q][H*d]  (A_full in dual mode)

@@ -142,6 +142,20 @@ def test_validation_errors_without_gpu():
     assert L.ispa_ls_solve(ctypes.byref(st), 16, 128, -1.0, 16, None, 16, 1 << 30, None) == abi.ISPA_ERR_INVALID_ARG
 
 
+def test_attention_option_validation_without_gpu():
+    L = abi.lib()
+    r = KVRing(2, 64, 16, 4, 0, 0, 2, 16, 16)
+    # unknown option bit
+    assert L.ispa_attn_full_ex(ctypes.byref(r), 16, 16, 16, 32, 0.0, 2, 16, None, None) == abi.ISPA_ERR_INVALID_ARG
+    # frame-causal needs whole chunk frames (n_q a multiple of tokens_per_frame = 16)
+    assert L.ispa_attn_full_ex(ctypes.byref(r), 16, 16, 16, 24, 0.0, abi.ISPA_ATTN_FRAME_CAUSAL, 16, None,
+                               None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_attn_local_ex(ctypes.byref(r), Window(0, 1), 16, 16, 16, 24, 0.0, abi.ISPA_ATTN_FRAME_CAUSAL,
+                                16, None, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_attn_dual_ex(ctypes.byref(r), Window(0, 1), 16, 16, 16, 32, 0.0, 4, 16, 16, 16, 16, None, None,
+                               16, 1 << 20, None) == abi.ISPA_ERR_INVALID_ARG
+
+
 def test_workspace_sizes():
     assert abi.ispa_attn_dual_workspace_size(12, 4680) == 12 * 4680 * 4
     assert abi.ispa_ls_state_bytes(1536) == 4 * 1536 * 1536 * 4

@@ -71,21 +71,24 @@ def test_empty_key_set():
     assert np.all(o == 0) and np.all(np.isneginf(lse))
 
 
-def _brute_force(q, k_hist, v_hist, k_cur, v_cur, P, member, scale):
+def _brute_force(q, k_hist, v_hist, k_cur, v_cur, P, member, scale, chunk_member=None):
     """Masked dense softmax written with Python loops and math.exp.
 
-    member(f) says whether past frame f is in the key set; chunk keys always are.
+    member(f) says whether past frame f is in the key set; chunk key j is in it for
+    query i when chunk_member(i, j) (always, by default).
     """
     nq, H, d = q.shape
     nh = k_hist.shape[0]
-    keys = [(j, k_hist[j], v_hist[j], member(j // P)) for j in range(nh)]
-    keys += [(nh + j, k_cur[j], v_cur[j], True) for j in range(k_cur.shape[0])]
+    keys = [(None, k_hist[j], v_hist[j], member(j // P)) for j in range(nh)]
+    keys += [(j, k_cur[j], v_cur[j], True) for j in range(k_cur.shape[0])]
     out = np.zeros((nq, H, d))
     lse = np.zeros((H, nq))
     for h in range(H):
         for i in range(nq):
             scores = []
-            for _, kk, _, use in keys:
+            for cj, kk, _, use in keys:
+                if cj is not None and chunk_member is not None:
+                    use = chunk_member(i, cj)
                 scores.append(scale * sum(float(q[i, h, c]) * float(kk[h, c]) for c in range(d))
                               if use else -math.inf)
             mx = max(scores)
@@ -193,3 +196,65 @@ def test_keysets_used_by_local_match_eq7():
     o_f, l_f = at.attn_full(s.q, s.k_hist, v_hist, s.k_cur, v_cur, P)
     _, l_l = at.attn_local(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, n_sink, n_recent)
     assert np.allclose(o_f[:, 0, 0], np.exp(l_l[0] - l_f[0]), atol=1e-13)
+
+
+# ------------------------------------------------------------------ frame-causal chunk option
+
+@pytest.mark.parametrize("n_sink,n_recent", [(0, 2), (1, 0)])
+def test_frame_causal_brute_force(n_sink, n_recent):
+    # query i of chunk frame i // P sees chunk key j iff j // P <= i // P (frames up to its own)
+    P, H, d, F = 3, 2, 4, 4
+    s = synth.make_step(12, F, P, H, d, n_chunk_frames=3)
+    scale = 1.0 / math.sqrt(d)
+    causal = lambda i, j: j // P <= i // P  # noqa: E731
+    o_f, l_f = at.attn_full(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, frame_causal=True)
+    b_f, bl_f = _brute_force(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, lambda f: True, scale, causal)
+    assert np.allclose(o_f, b_f, atol=1e-12) and np.allclose(l_f, bl_f, atol=1e-12)
+    o_l, l_l = at.attn_local(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, n_sink, n_recent,
+                             frame_causal=True)
+    b_l, bl_l = _brute_force(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P,
+                             lambda f: f < n_sink or f >= F - n_recent, scale, causal)
+    assert np.allclose(o_l, b_l, atol=1e-12) and np.allclose(l_l, bl_l, atol=1e-12)
+
+
+def test_frame_causal_special_cases():
+    P, H, d, F = 5, 2, 8, 3
+    s = synth.make_step(13, F, P, H, d, n_chunk_frames=3)
+    dense, ld = at.attn_full(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P)
+    causal, lc = at.attn_full(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, frame_causal=True)
+    # the chunk's last frame sees the whole chunk: identical to the dense chunk
+    assert np.array_equal(causal[2 * P:], dense[2 * P:]) and np.array_equal(lc[:, 2 * P:], ld[:, 2 * P:])
+    # earlier frames do differ
+    assert np.abs(causal[:P] - dense[:P]).max() > 1e-3
+    # no past, chunk frame 0: plain attention over the chunk's first frame
+    s0 = synth.make_step(14, 0, P, H, d, n_chunk_frames=3)
+    o0, _ = at.attn_full(s0.q, s0.k_hist, s0.v_hist, s0.k_cur, s0.v_cur, P, frame_causal=True)
+    want, _ = at.attend_heads(s0.q[:P], s0.k_cur[:P], s0.v_cur[:P], 1.0 / math.sqrt(d))
+    assert np.allclose(o0[:P], want, atol=1e-13)
+    # a one-frame chunk is unchanged by the option
+    s1 = synth.make_step(15, F, P, H, d, n_chunk_frames=1)
+    a, _ = at.attn_full(s1.q, s1.k_hist, s1.v_hist, s1.k_cur, s1.v_cur, P)
+    b, _ = at.attn_full(s1.q, s1.k_hist, s1.v_hist, s1.k_cur, s1.v_cur, P, frame_causal=True)
+    assert np.array_equal(a, b)
+    # row subsets stay exact
+    rows = np.array([0, 4, 7, 11, 14])
+    sub, lsub = at.attn_full(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, rows=rows, frame_causal=True)
+    assert np.allclose(sub, causal[rows], atol=1e-14) and np.allclose(lsub, lc[:, rows], atol=1e-14)
+
+
+def test_frame_causal_fusion_identity():
+    # Eq. 11-12 still reconstruct the full set: history frames are past frames, unmasked
+    P, H, d, F = 4, 2, 8, 7
+    s = synth.make_step(16, F, P, H, d, n_chunk_frames=3)
+    loc, ll = at.attn_local(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, 1, 2, frame_causal=True)
+    hist, lh = at.attn_hist(s.q, s.k_hist, s.v_hist, P, 1, 2)
+    fused, lf = at.lse_fuse(loc, ll, hist, lh)
+    full, lfull = at.attn_full(s.q, s.k_hist, s.v_hist, s.k_cur, s.v_cur, P, frame_causal=True)
+    assert np.allclose(fused, full, atol=1e-12) and np.allclose(lf, lfull, atol=1e-12)
+
+
+def test_frame_causal_needs_whole_frames():
+    P, H, d = 4, 1, 4
+    s = synth.make_step(17, 2, P, H, d, n_chunk_frames=2)
+    with pytest.raises(ValueError):
+        at.attn_full(s.q[:6], s.k_hist, s.v_hist, s.k_cur[:6], s.v_cur[:6], P, frame_causal=True)
