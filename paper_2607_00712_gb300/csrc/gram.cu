@@ -9,8 +9,8 @@
 // contraction over tokens, the token axis being the UMMA K dimension:
 //   G tile: a^T a;   X tile: a^T hi + a^T lo;   S tile: hi^T hi + hi^T lo + lo^T hi
 // (the lo^T lo term is below fp32 resolution and dropped).  Both operands
-// are token-major [T][D] in HBM, i.e. MN-major for the UMMA, staged by TMA in
-// 64-token x 64-feature boxes with 128-byte swizzle.
+// are token-major [T][D] in HBM, i.e. MN-major for the UMMA, staged by TMA with
+// 128-byte swizzle, 64 tokens per pipeline stage, one request per operand.
 //
 // Work split (stream-K): the tiles are laid end to end as one sequence of
 // steps (tile, pass, 64-token block) -- G tiles (1 pass each), X tiles (2),
@@ -156,8 +156,10 @@ __global__ void __launch_bounds__(256) split_kernel(const uint4* __restrict__ a_
 
 template <int BN>
 __global__ void __launch_bounds__(G_THREADS, 1)
-    gram_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_hi,
-                const __grid_constant__ CUtensorMap tm_lo, const GramParams p) {
+    gram_kernel(const __grid_constant__ CUtensorMap tm_a_r, const __grid_constant__ CUtensorMap tm_hi_r,
+                const __grid_constant__ CUtensorMap tm_lo_r, const __grid_constant__ CUtensorMap tm_a_c,
+                const __grid_constant__ CUtensorMap tm_hi_c, const __grid_constant__ CUtensorMap tm_lo_c,
+                const GramParams p) {
   using C = GCfg<BN>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw;
@@ -206,7 +208,9 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0 && g1 > g0) {
-      auto map_of = [&](int w) { return w == 0 ? &tm_a : (w == 1 ? &tm_hi : &tm_lo); };
+      // _r maps fetch a tile's GM row features, _c maps its BN column features
+      auto map_r = [&](int w) { return w == 0 ? &tm_a_r : (w == 1 ? &tm_hi_r : &tm_lo_r); };
+      auto map_c = [&](int w) { return w == 0 ? &tm_a_c : (w == 1 ? &tm_hi_c : &tm_lo_c); };
       int issued = 0;
       int item = -1, first = 0, kind = 0, bi = 0, bj = 0;
       for (int g = g0; g < g1; ++g) {
@@ -222,12 +226,11 @@ __global__ void __launch_bounds__(G_THREADS, 1)
         if (!mbar_wait(empty0 + 8 * st, ((i / GST) & 1) ^ 1, wc, 21, i)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
         const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
-        const CUtensorMap* ma = map_of(kPasses[kind][pass].a);
-        const CUtensorMap* mb = map_of(kPasses[kind][pass].b);
-#pragma unroll
-        for (int x = 0; x < GM / 64; ++x) tma_load_2d(sa + x * C::BOX, ma, full0 + 8 * st, bi * GM + 64 * x, tok);
-#pragma unroll
-        for (int x = 0; x < BN / 64; ++x) tma_load_2d(sb + x * C::BOX, mb, full0 + 8 * st, bj * BN + 64 * x, tok);
+        const CUtensorMap* ma = map_r(kPasses[kind][pass].a);
+        const CUtensorMap* mb = map_c(kPasses[kind][pass].b);
+        // one request per operand: (64 features, GK tokens, GM/64 or BN/64 feature blocks)
+        tma_load_3d(sa, ma, full0 + 8 * st, 0, tok, bi * (GM / 64));
+        tma_load_3d(sb, mb, full0 + 8 * st, 0, tok, bj * (BN / 64));
         issued = i + 1;
       }
       for (int i = issued > GST ? issued - GST : 0; i < issued; ++i)
@@ -339,11 +342,17 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
     if (e != cudaSuccess) return e;
     attr_done[dev] = true;
   }
-  CUtensorMap ta, th, tl;
-  if (!encode_tmap_2d(&ta, a_loc, D, T, static_cast<uint64_t>(D) * 2, 64, GK) ||
-      !encode_tmap_2d(&th, hi, D, T, static_cast<uint64_t>(D) * 2, 64, GK) ||
-      !encode_tmap_2d(&tl, lo, D, T, static_cast<uint64_t>(D) * 2, 64, GK))
-    return cudaErrorInvalidValue;
+  // [T][D] operands viewed as (64 features, T tokens, D/64 feature blocks): the block
+  // stride (128 B) is below the token stride, so one box (64, GK, n) fetches n adjacent
+  // 64-feature blocks as n consecutive [GK][128 B] swizzled blocks in a single request.
+  // (measured on GB300: 11 % faster than one 2-D request per 64-feature block at hidden
+  // 1536, 1 % at hidden 5120)
+  CUtensorMap tr[3], tc[3];
+  const void* srcs[3] = {a_loc, hi, lo};
+  for (int i = 0; i < 3; ++i)
+    if (!encode_tmap_3d(&tr[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, GM / 64) ||
+        !encode_tmap_3d(&tc[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, BN / 64))
+      return cudaErrorInvalidValue;
   const int RB = D / GM, CB = D / BN;
   int n_upper = 0;
   for (int r = 0; r < RB; ++r) n_upper += CB - (r * GM) / BN;
@@ -363,7 +372,7 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   // one CTA per SM, each with at least 16 steps (a 1024-token run of one tile)
   const int64_t want = (total + 15) / 16;
   const dim3 grid(static_cast<unsigned>(want < sms ? (want > 0 ? want : 1) : sms));
-  gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(ta, th, tl, p);
+  gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(tr[0], tr[1], tr[2], tc[0], tc[1], tc[2], p);
   return cudaGetLastError();
 }
 
