@@ -194,10 +194,19 @@ class StepRunner:
         self.launches_per_step = 7   # 3 attention + disc reduce + split + gram + append
         torch.cuda.synchronize(device)
 
-    def step(self, ev=None):
-        """Enqueue one step; ev = list of 6 events to record between the calls (or None)."""
+    def outputs(self):
+        """The step's result tensors (the ones an e2e run reads back)."""
+        return [self.out_full, self.out_local, self.a_full, self.a_loc, self.disc]
+
+    def step(self, ev=None, inputs=None, outs=None):
+        """Enqueue one step; ev = list of 6 events to record between the calls (or None).
+
+        inputs / outs: another set of (q, k_cur, v_cur) triples / result tensors of the same
+        shapes (the e2e pipeline alternates two sets); default: the runner's own."""
         abi, nq = self.abi, self.wl["nq"]
         s = self.stream
+        inputs = self.inputs if inputs is None else inputs
+        out_full, out_local, a_full, a_loc, disc = self.outputs() if outs is None else outs
         if self.debug:
             def rec(i):
                 self.torch.cuda.synchronize()
@@ -206,21 +215,21 @@ class StepRunner:
         else:
             rec = (lambda i: ev[i].record(s)) if ev else (lambda i: None)
         rec(0)
-        q, kc, vc = self.inputs[0]
-        abi.ispa_attn_full(self.rings[0].c, q, kc, vc, nq, 0.0, self.out_full, None, s)
+        q, kc, vc = inputs[0]
+        abi.ispa_attn_full(self.rings[0].c, q, kc, vc, nq, 0.0, out_full, None, s)
         rec(1)
-        q, kc, vc = self.inputs[1]
-        abi.ispa_attn_local(self.rings[1].c, self.win, q, kc, vc, nq, 0.0, self.out_local, None, s)
+        q, kc, vc = inputs[1]
+        abi.ispa_attn_local(self.rings[1].c, self.win, q, kc, vc, nq, 0.0, out_local, None, s)
         rec(2)
-        q, kc, vc = self.inputs[2]
-        abi.ispa_attn_dual(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, self.a_full, self.a_loc, self.disc,
+        q, kc, vc = inputs[2]
+        abi.ispa_attn_dual(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, a_full, a_loc, disc,
                            self.disc_sum, None, None, self.dual_ws, self.dual_wsb, s)
         rec(3)
-        abi.ispa_ls_accumulate(self.ls.c, self.a_loc, self.a_full, nq, self.ls_ws, self.ls_wsb, s)
+        abi.ispa_ls_accumulate(self.ls.c, a_loc, a_full, nq, self.ls_ws, self.ls_wsb, s)
         rec(4)
         for i in range(3):
             self.ring_arr[i] = self.rings[i].c
-        abi.ispa_kv_append_layers(self.ring_arr, [x[1] for x in self.inputs], [x[2] for x in self.inputs],
+        abi.ispa_kv_append_layers(self.ring_arr, [x[1] for x in inputs], [x[2] for x in inputs],
                                   self.wl["L"], s)
         for i in range(3):
             self.rings[i].c.frames_written = self.ring_arr[i].frames_written
@@ -382,34 +391,66 @@ def run_extras(r, wl, device, reps=20):
 
 
 def run_e2e(r, args, device, flops_step, world):
-    """The same step through the C-ABI with pinned host inputs / outputs copied inside the timed region."""
+    """The same step through the C-ABI with pinned host inputs / outputs copied inside the timed region.
+
+    Every step copies its own inputs host->device before its compute and reads its results
+    device->host after it.  The copies of step i+1 (in) and i-1 (out) run on two copy streams
+    while step i computes: two sets of device inputs and outputs alternate, ordered by events
+    (step i's inputs land before it starts; a set is refilled only after the step that used it
+    has finished computing and has been read back).  Timed from the first copy in to the last
+    copy out, divided by the number of steps.
+    """
     import torch
     host_in = [[t.cpu().pin_memory() for t in trip] for trip in r.inputs]
-    outs = [r.out_full, r.out_local, r.a_full, r.a_loc, r.disc]
-    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs]
+    dev_in = [r.inputs, [tuple(torch.empty_like(t) for t in trip) for trip in r.inputs]]
+    dev_out = [r.outputs(), [torch.empty_like(t) for t in r.outputs()]]
+    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in r.outputs()]
     h2d = sum(t.numel() * t.element_size() for trip in host_in for t in trip)
     d2h = sum(t.numel() * t.element_size() for t in host_out)
-    s = r.stream
+    s_comp = r.stream
+    s_in, s_out = torch.cuda.Stream(device), torch.cuda.Stream(device)
     n = max(3, min(args.steps, 20))
 
-    def one():
-        for trip_h, trip_d in zip(host_in, r.inputs):
-            for h, dv in zip(trip_h, trip_d):
-                dv.copy_(h, non_blocking=True)
-        r.step()
-        for h, dv in zip(host_out, outs):
-            h.copy_(dv, non_blocking=True)
-    one()
+    def run(steps, e_start=None, e_end=None):
+        ev_comp, ev_out = [], []
+        for i in range(steps):
+            b = i % 2
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(ev_comp[i - 2])          # set b no longer read by step i-2
+                if i == 0 and e_start is not None:
+                    e_start.record(s_in)
+                for trip_h, trip_d in zip(host_in, dev_in[b]):
+                    for h, dv in zip(trip_h, trip_d):
+                        dv.copy_(h, non_blocking=True)
+                e_in = torch.cuda.Event()
+                e_in.record(s_in)
+            s_comp.wait_event(e_in)
+            if i >= 2:
+                s_comp.wait_event(ev_out[i - 2])             # outputs of set b read back
+            r.step(inputs=dev_in[b], outs=dev_out[b])
+            e_c = torch.cuda.Event()
+            e_c.record(s_comp)
+            ev_comp.append(e_c)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(e_c)
+                for h, dv in zip(host_out, dev_out[b]):
+                    h.copy_(dv, non_blocking=True)
+                e_o = torch.cuda.Event()
+                e_o.record(s_out)
+                ev_out.append(e_o)
+        if e_end is not None:
+            e_end.record(s_out)
+
+    run(2)
     torch.cuda.synchronize(device)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(s)
-    for _ in range(n):
-        one()
-    e1.record(s)
+    run(n, e0, e1)
     torch.cuda.synchronize(device)
     ms = e0.elapsed_time(e1) / n
     return dict(value=round(world * flops_step / (ms * 1e-3) / 1e12, 3), unit=UNIT, h2d_bytes_per_step=h2d,
-                d2h_bytes_per_step=d2h, ms_per_step=round(ms, 4), steps=n)
+                d2h_bytes_per_step=d2h, ms_per_step=round(ms, 4), steps=n,
+                overlap="copies on two streams, double-buffered device inputs and outputs")
 
 
 # ---------------------------------------------------------------- oracle legs
