@@ -15,6 +15,9 @@ Modules
                outputs and their discrepancy, and the LSE fusion (Eq. 9-12).
   ls        -- accumulation of the normal-equation sums, the textbook
                Cholesky solve of Eq. 5 and the feasibility score of Eq. 6.
+  quant     -- e4m3 coding from the format definition, per-token / per-channel
+               quantisation and the W8A8 linear layer on W + dW (Sec. 4's
+               post-training quantisation).
 
 Every function runs in float64.  Pins (what each function is checked
 against, independent of itself) live in tests/test_oracle_*.py.
