@@ -387,7 +387,57 @@ def run_extras(r, wl, device, reps=20):
         out["ls_solve_dim"] = D
     except abi.IspaError as e:
         out["ls_solve_error"] = str(e)
+        dW.zero_()
+    out.update(run_w8a8(r, wl, device, W, dW, reps))
     return out
+
+
+def run_w8a8(r, wl, device, W, dW, reps):
+    """The attention output projection with 8-bit weights and activations (Sec. 4) on the
+    injected weight W + dW: weight quantisation (once per transition), then per step the
+    activation quantisation and the e4m3 GEMM, next to a cuBLAS bf16 GEMM of the same shape
+    (context for the latency breakdown).  Inputs stay L2-warm across the repetitions."""
+    import torch
+    abi = r.abi
+    T, D = wl["nq"], wl["D"]
+    a = r.a_full                                   # [T][D] bf16, a real attention output
+    wq = torch.empty(D, D, dtype=torch.uint8, device=device)
+    ws = torch.empty(D, dtype=torch.float32, device=device)
+    aq = torch.empty(T, D, dtype=torch.uint8, device=device)
+    sa = torch.empty(T, dtype=torch.float32, device=device)
+    y = torch.empty(T, D, dtype=torch.bfloat16, device=device)
+    s = r.stream
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev[0].record(s)
+    abi.ispa_quantize_weight_e4m3(W, dW, D, D, wq, ws, s)
+    ev[1].record(s)
+    torch.cuda.synchronize(device)
+    t_wq = ev[0].elapsed_time(ev[1])
+    w_bf16 = (W + dW).to(torch.bfloat16)
+    t_q = t_mm = t_ref = 0.0
+    for i in range(reps + 3):
+        ev[0].record(s)
+        abi.ispa_quantize_rows_e4m3(a, T, D, aq, sa, s)
+        ev[1].record(s)
+        abi.ispa_linear_w8a8(aq, sa, wq, ws, T, D, D, y, s)
+        ev[2].record(s)
+        torch.matmul(a, w_bf16)
+        ev[3].record(s)
+        torch.cuda.synchronize(device)
+        if i >= 3:
+            t_q += ev[0].elapsed_time(ev[1])
+            t_mm += ev[1].elapsed_time(ev[2])
+            t_ref += ev[2].elapsed_time(ev[3])
+    t_q, t_mm, t_ref = t_q / reps, t_mm / reps, t_ref / reps
+    flops = 2.0 * T * D * D
+    pk = peaks()
+    fp8_peak = 2.0 * pk["bf16"]                    # measured bf16 peak x the nominal fp8 / bf16 ratio
+    tf = flops / (t_mm * 1e-3) / 1e12
+    return dict(w8a8_weight_quant_ms=round(t_wq, 4), w8a8_act_quant_ms=round(t_q, 4),
+                w8a8_gemm_ms=round(t_mm, 4), w8a8_gemm_tflops=round(tf, 1),
+                w8a8_gemm_frac_of_fp8_peak=round(tf / fp8_peak, 4), w8a8_fp8_peak_tflops=fp8_peak,
+                cublas_bf16_projection_ms=round(t_ref, 4),
+                w8a8_shape=f"{T} x {D} -> {D}")
 
 
 def run_e2e(r, args, device, flops_step, world):

@@ -408,6 +408,39 @@ ISPA_API ispa_status ispa_ls_solve(const ispa_ls_state* state, const float* W, i
                           double lambda, float* dW, double* eps_out, void* workspace,
                           size_t ws_bytes, ispa_stream stream);
 
+/* ------------------------------------------------------------ W8A8 projection */
+/*
+ * 8-bit weights and activations for the attention output projection on the
+ * injected weight W + dW (Sec. 4 runs ISPA with W8A8 linear layers; Sec. 3.2
+ * gives W_new = W + dW).  The paper fixes no 8-bit format; here it is fp8 e4m3
+ * ("fn": largest magnitude 448, no infinities) with one fp32 scale per token
+ * for activations and one per output channel for weights:
+ *   amax = max |x| over the group; inv = 448 / amax and scale = amax / 448 in
+ *   fp32 (both 1 for an all-zero group); code = e4m3(x * inv), rounded to
+ *   nearest even and saturated at +-448.
+ */
+
+/* Activations x: bf16 [rows][cols] -> codes q: uint8 [rows][cols], scale: fp32
+ * [rows].  cols % 16 == 0 (else ISPA_ERR_UNSUPPORTED); x and q 16-byte aligned. */
+ISPA_API ispa_status ispa_quantize_rows_e4m3(const void* x, int64_t rows, int32_t cols, uint8_t* q,
+                                             float* scale, ispa_stream stream);
+
+/* Weight W (+ dW, nullable): fp32 [D][D_out] (row-vector convention y = a W) ->
+ * codes q_t: uint8 [D_out][D] (K-major, the layout of a Linear weight) and
+ * scale: fp32 [D_out], one per output channel of W + dW (summed in fp32).
+ * D % 16 == 0.  Three launches; once per weight update, not per step. */
+ISPA_API ispa_status ispa_quantize_weight_e4m3(const float* W, const float* dW, int32_t D, int32_t D_out,
+                                               uint8_t* q_t, float* scale, ispa_stream stream);
+
+/* out: bf16 [T][D_out] = a_scale[t] * w_scale[n] * sum_k dec(a_q[t][k]) * dec(w_q[n][k]),
+ * with a_q [T][D] and w_q [D_out][D] e4m3 codes from the two calls above, fp32
+ * accumulation on the tensor cores, bf16 output (round to nearest).
+ * D % 128 == 0 and D_out % 128 == 0 (else ISPA_ERR_UNSUPPORTED); a_q, w_q, out
+ * 16-byte aligned. */
+ISPA_API ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uint8_t* w_q,
+                                      const float* w_scale, int64_t T, int32_t D, int32_t D_out, void* out,
+                                      ispa_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -110,6 +110,10 @@ _SIGS = {
     "ispa_ls_accumulate": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
                                      c_void_p]),
     "ispa_ls_solve_workspace_size": (c_size_t, [c_int32, c_int32]),
+    "ispa_quantize_rows_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_quantize_weight_e4m3": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_linear_w8a8": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_int32, c_int32, c_void_p,
+                                   c_void_p]),
     "ispa_ls_solve": (c_int32, [POINTER(LSState), c_void_p, c_int32, c_double, c_void_p, POINTER(c_double),
                                 c_void_p, c_size_t, c_void_p]),
 }
@@ -323,3 +327,20 @@ def ispa_ls_solve(state: LSState, W, d_out: int, lam: float, dW, workspace, ws_b
     _check(lib().ispa_ls_solve(ctypes.byref(state), _ptr(W), d_out, lam, _ptr(dW), ctypes.byref(eps),
                                _ptr(workspace), ws_bytes, _stream(stream)), "ispa_ls_solve")
     return eps.value
+
+
+# ---------------------------------------------------------------- W8A8 projection
+def ispa_quantize_rows_e4m3(x, rows: int, cols: int, q, scale, stream=None) -> None:
+    _check(lib().ispa_quantize_rows_e4m3(_ptr(x), rows, cols, _ptr(q), _ptr(scale), _stream(stream)),
+           "ispa_quantize_rows_e4m3")
+
+
+def ispa_quantize_weight_e4m3(W, dW, D: int, D_out: int, q_t, scale, stream=None) -> None:
+    _check(lib().ispa_quantize_weight_e4m3(_ptr(W), _ptr(dW), D, D_out, _ptr(q_t), _ptr(scale), _stream(stream)),
+           "ispa_quantize_weight_e4m3")
+
+
+def ispa_linear_w8a8(a_q, a_scale, w_q, w_scale, T: int, D: int, D_out: int, out, stream=None) -> None:
+    _check(lib().ispa_linear_w8a8(_ptr(a_q), _ptr(a_scale), _ptr(w_q), _ptr(w_scale), T, D, D_out, _ptr(out),
+                                  _stream(stream)), "ispa_linear_w8a8")
+

@@ -108,6 +108,19 @@ bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], c
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
+                       uint32_t b0, uint32_t b1) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {d0, d1};
+  cuuint64_t strides[1] = {stride1_bytes};
+  cuuint32_t box[2] = {b0, b1};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1) {
   EncodeTiledFn fn = encode_fn();
@@ -557,5 +570,38 @@ ispa_status ispa_ls_solve(const ispa_ls_state* st, const float* W, int32_t d_out
   if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
   return run_ls_solve(st->dim, st->gram, W, d_out, lambda, dW, eps_out, workspace, stream);
 }
+
+// ------------------------------------------------------------ W8A8 projection (Sec. 4)
+
+ispa_status ispa_quantize_rows_e4m3(const void* x, int64_t rows, int32_t cols, uint8_t* q, float* scale,
+                                    ispa_stream stream) {
+  if (!x || !q || !scale || rows <= 0 || cols <= 0 || !aligned16(x) || !aligned16(q)) return ISPA_ERR_INVALID_ARG;
+  if (cols % 16 != 0) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_rows(x, rows, cols, q, scale, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_quantize_weight_e4m3(const float* W, const float* dW, int32_t D, int32_t D_out, uint8_t* q_t,
+                                      float* scale, ispa_stream stream) {
+  if (!W || !q_t || !scale || D <= 0 || D_out <= 0 || !aligned16(q_t)) return ISPA_ERR_INVALID_ARG;
+  if (D % 16 != 0) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_weight(W, dW, D, D_out, q_t, scale, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uint8_t* w_q, const float* w_scale,
+                             int64_t T, int32_t D, int32_t D_out, void* out, ispa_stream stream) {
+  if (!a_q || !a_scale || !w_q || !w_scale || !out || T <= 0 || T > INT32_MAX || D <= 0 || D_out <= 0 ||
+      !aligned16(a_q) || !aligned16(w_q) || !aligned16(out))
+    return ISPA_ERR_INVALID_ARG;
+  if (D % 128 != 0 || D_out % 128 != 0) return ISPA_ERR_UNSUPPORTED;
+  int* status = device_status_ptr();
+  if (!status) return ISPA_ERR_CUDA;
+  if (launch_w8a8_gemm(a_q, a_scale, w_q, w_scale, static_cast<int32_t>(T), D, D_out, out, status, g_wait_limit,
+                       stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
 
 }  // extern "C"

@@ -92,6 +92,14 @@ size_t ls_solve_ws_bytes(int32_t D, int32_t d_out);
 ispa_status run_ls_solve(int32_t D, const float* gram, const float* W, int32_t d_out,
                          double lambda, float* dW, double* eps_out, void* ws, cudaStream_t s);
 
+// ------------------------------------------------------------ W8A8 projection
+cudaError_t launch_quant_rows(const void* x, int64_t rows, int32_t cols, uint8_t* q, float* scale, cudaStream_t s);
+cudaError_t launch_quant_weight(const float* W, const float* dW, int32_t D, int32_t Dout, uint8_t* q_t, float* scale,
+                                cudaStream_t s);
+cudaError_t launch_w8a8_gemm(const uint8_t* a_q, const float* a_scale, const uint8_t* w_q, const float* w_scale,
+                             int32_t T, int32_t D, int32_t Dout, void* out, int* status, uint64_t wait_limit_ns,
+                             cudaStream_t s);
+
 // ------------------------------------------------------------ misc
 int* device_status_ptr();  // library status word on the current device (nullptr on error)
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
@@ -102,6 +110,9 @@ bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], c
                     const uint32_t box4[4]);
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
+// uint8 elements, 128-byte swizzle, rank 2.
+bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
+                       uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();
 uint32_t* next_heartbeat_slot(uint32_t kernel_tag);  // null unless a heartbeat buffer is set
 uint64_t* trace_buffer(int32_t* n_tiles);            // null unless a trace buffer is set

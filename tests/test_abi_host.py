@@ -156,6 +156,18 @@ def test_attention_option_validation_without_gpu():
                                16, 1 << 20, None) == abi.ISPA_ERR_INVALID_ARG
 
 
+def test_w8a8_validation_without_gpu():
+    L = abi.lib()
+    assert L.ispa_linear_w8a8(16, 16, 16, 16, 100, 192, 256, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D % 128
+    assert L.ispa_linear_w8a8(16, 16, 16, 16, 100, 256, 192, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D_out % 128
+    assert L.ispa_linear_w8a8(16, 16, 16, 16, 0, 256, 256, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_linear_w8a8(24, 16, 16, 16, 10, 256, 256, 16, None) == abi.ISPA_ERR_INVALID_ARG    # misaligned
+    assert L.ispa_quantize_rows_e4m3(16, 10, 24, 16, 16, None) == abi.ISPA_ERR_UNSUPPORTED           # cols % 16
+    assert L.ispa_quantize_rows_e4m3(None, 10, 32, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_quantize_weight_e4m3(16, None, 24, 32, 16, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D % 16
+    assert L.ispa_quantize_weight_e4m3(16, None, 32, 0, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
+
+
 def test_workspace_sizes():
     assert abi.ispa_attn_dual_workspace_size(12, 4680) == 12 * 4680 * 4
     assert abi.ispa_ls_state_bytes(1536) == 4 * 1536 * 1536 * 4
