@@ -20,6 +20,11 @@ Quantisation, in fp32 as both sides compute it:
   else inv = fl32(448 / amax), scale = fl32(amax / 448); code = e4m3(fl32(x * inv)).
 Linear: y[t, n] = a_scale[t] * w_scale[n] * sum_k dec(a_q[t, k]) * dec(w_q[n, k]), in float64
 (the weight codes are stored K-major, [D_out][D]).
+
+8-bit query/key attention (SageAttention's 8-bit Q K^T with 16-bit P V, cited in Sec. 3.4):
+one scale per head, scale = fl32(amax / 448) over all the group's tokens (or a given scale, for
+keys appended into a cache), code = e4m3(fl32(x / scale)); the attention is then the plain
+attention of the dequantised q and k (codes times scale) with the unquantised v.
 """
 from __future__ import annotations
 
@@ -103,3 +108,29 @@ def linear_w8a8(a_q, a_scale, w_q, w_scale) -> np.ndarray:
     Wt = decode(w_q)
     acc = A @ Wt.T
     return acc * np.asarray(a_scale, np.float64)[:, None] * np.asarray(w_scale, np.float64)[None, :]
+
+
+def quantize_heads_with_scale(x, scale) -> np.ndarray:
+    """Token-major [n][H][d] values and per-head scales [H] -> codes e4m3(fl32(x / scale_h))."""
+    x = np.asarray(x, dtype=np.float32)
+    s = np.asarray(scale, dtype=np.float32)[None, :, None]
+    return encode((x / s).astype(np.float32))
+
+
+def head_scales(x) -> np.ndarray:
+    """Per-head scale fl32(amax / 448) of token-major [n][H][d] values (1 for an all-zero head)."""
+    x = np.asarray(x, dtype=np.float32)
+    amax = np.max(np.abs(x), axis=(0, 2)).astype(np.float32)
+    return np.where(amax == 0, np.float32(1), amax / np.float32(E4M3_MAX)).astype(np.float32)
+
+
+def quantize_heads(x):
+    """[n][H][d] -> (codes, per-head scales [H])."""
+    s = head_scales(x)
+    return quantize_heads_with_scale(x, s), s
+
+
+def dequantize_heads(q, scale) -> np.ndarray:
+    """codes [n][H][d], scales [H] -> float64 values."""
+    return decode(q) * np.asarray(scale, np.float64)[None, :, None]
+

@@ -120,3 +120,26 @@ def test_linear_identity_weight_returns_dequantised_activations():
     assert np.all(sw == np.float32(1 / 448)) and np.all(qt.decode(np.diag(wq)) == 448.0)
     y = qt.linear_w8a8(aq, sa, wq, sw)
     assert np.allclose(y, qt.decode(aq) * sa[:, None], rtol=1e-6, atol=0)
+
+
+def test_head_quantisation_and_dequantisation():
+    r = np.random.default_rng(6)
+    x = (r.standard_normal((50, 3, 16)) * np.array([0.1, 3.0, 40.0])[None, :, None]).astype(np.float32)
+    x[:, 1, :] = 0.0                                     # an all-zero head
+    q, s = qt.quantize_heads(x)
+    assert s.dtype == np.float32 and s[1] == 1.0 and np.all(q[:, 1, :] == 0)
+    amax = np.abs(x).max(axis=(0, 2))
+    assert s[0] == np.float32(amax[0]) / np.float32(448) and s[2] == np.float32(amax[2]) / np.float32(448)
+    back = qt.dequantize_heads(q, s)
+    err = np.abs(back - x)
+    assert np.all(err <= 2.0 ** -4 * np.abs(x) * (1 + 1e-6) + 2.0 ** -10 * s[None, :, None])
+    # the largest magnitude of a head maps to (about) +-448: within one rounding of the division
+    for h in (0, 2):
+        i = np.unravel_index(np.argmax(np.abs(x[:, h, :])), x[:, h, :].shape)
+        assert abs(qt.decode(q[i[0], h, i[1]])) in (416.0, 448.0)
+
+
+def test_quantize_with_scale_saturates_outliers():
+    x = np.array([[[1.0, -2.0, 1000.0, -1e6]]], dtype=np.float32)
+    q = qt.quantize_heads_with_scale(x, np.array([1.0], np.float32))
+    assert list(qt.decode(q).ravel()) == [1.0, -2.0, 448.0, -448.0]
