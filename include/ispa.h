@@ -68,17 +68,23 @@ typedef enum {
  *   overwrites the oldest non-sink frame.  frames_written counts the frames
  *   appended so far; it is advanced on the host by ispa_kv_append when the
  *   copy is enqueued.  The struct is plain data: copying it (and the two
- *   buffers) checkpoints the cache.  Slots never written must still hold
+ *   buffers) checkpoints the cache.  With k_format = ISPA_KV_K_E4M3, k holds
+ *   e4m3 codes [H][capacity_frames * P][head_dim] (one byte each; head_dim 128)
+ *   written by ispa_kv_append_qk8 with one fp32 scale per head that the caller
+ *   keeps for the ring's life.  Slots never written must still hold
  *   finite values (zero-fill the buffers at creation): a key tile that ends
  *   inside a run reads the rows after it with weight zero, and 0 * NaN is NaN.
  */
+#define ISPA_KV_BF16 0     /* k_format: keys bf16 (every entry point except *_qk8) */
+#define ISPA_KV_K_E4M3 1   /* k_format: keys e4m3 codes, 1 byte each (the *_qk8 entry points) */
+
 typedef struct {
   int32_t num_heads;
   int32_t head_dim;
   int32_t tokens_per_frame;
   int32_t capacity_frames;
   int32_t n_sink_frames;
-  int32_t reserved;
+  int32_t k_format;       /* ISPA_KV_BF16 or ISPA_KV_K_E4M3; values stay bf16 */
   int64_t frames_written;
   void* k;
   void* v;
@@ -170,7 +176,8 @@ ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slot
  * next-S-issued, 6-7 TMA K / V issued).  NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
 
-/* Bytes of one ring's K and V buffers together (2 * H * cap * P * d * 2). */
+/* Bytes of one ring's K and V buffers together: H * cap * P * d * (2 + 2), or
+ * * (1 + 2) with e4m3 keys. */
 ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);
 
 /* Host-only: ring slot of logical frame `frame` (see ispa_kv_ring), or -1 if
@@ -407,6 +414,60 @@ ISPA_API size_t ispa_ls_solve_workspace_size(int32_t dim, int32_t d_out);
 ISPA_API ispa_status ispa_ls_solve(const ispa_ls_state* state, const float* W, int32_t d_out,
                           double lambda, float* dW, double* eps_out, void* workspace,
                           size_t ws_bytes, ispa_stream stream);
+
+/* ------------------------------------------------------------ 8-bit Q K^T attention */
+/*
+ * The chunk attention with queries and keys as fp8 e4m3 codes and values,
+ * probabilities and output as in the bf16 path -- the 8-bit Q K^T / 16-bit P V
+ * split of SageAttention, which the paper cites for its attention (Sec. 3.4).
+ * One fp32 scale per head: x ~ code * scale.  The result is the attention of
+ * the dequantised q and k (Eq. 3 / Eq. 7 on them), computed like the bf16 path.
+ * Head dim 128 only.
+ */
+
+/* x: bf16 [n][H][d] -> codes q: uint8 [n][H][d] and scale: fp32 [H] (written),
+ * scale_h = max |x_h| / 448 (1 for an all-zero head), code = e4m3(x * (1 / scale_h))
+ * (each step in fp32, rounded to nearest even), saturating.  d % 16 == 0, H <= 256. */
+ISPA_API ispa_status ispa_quantize_heads_e4m3(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q,
+                                              float* scale, ispa_stream stream);
+
+/* Queries for the *_qk8 attention: x bf16 [n][H][d] -> codes q [n][H][d] and
+ * scale fp32 [H][ceil(n / 128)] (written): one scale per head and block of 128
+ * consecutive tokens (the attention's query tile), computed like
+ * ispa_quantize_heads_e4m3 within each block.  d % 16 == 0, d <= 256. */
+ISPA_API ispa_status ispa_quantize_q_e4m3(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q,
+                                          float* scale, ispa_stream stream);
+
+/* Codes with given per-head scales: x bf16 [n][H][d], scale fp32 [H] (device)
+ * -> q [n][H][d], code = e4m3(x * (1 / scale_h)).  For the chunk's keys, with
+ * the ring's key scales.  d % 16 == 0. */
+ISPA_API ispa_status ispa_quantize_k_e4m3(const void* x, int64_t n, int32_t H, int32_t d, const float* scale,
+                                          uint8_t* q, ispa_stream stream);
+
+/* ispa_kv_append for a ring with k_format = ISPA_KV_K_E4M3: keys are coded
+ * with the ring's per-head scales k_scale[H] (device fp32, chosen by the caller
+ * once for the ring's life, e.g. from the first chunk's ispa_quantize_heads_e4m3;
+ * code = e4m3(k * (1 / scale)) as there; larger magnitudes saturate at
+ * +-448 * scale), values are copied as bf16. */
+ISPA_API ispa_status ispa_kv_append_qk8(ispa_kv_ring* ring, const void* k_new, const void* v_new,
+                                        int32_t n_frames, const float* k_scale, ispa_stream stream);
+
+/* ispa_attn_full / ispa_attn_local over a ring with e4m3 keys:
+ *   q8     : uint8 [n_q][H][128] codes, q_scale fp32 [H][ceil(n_q / 128)] (from
+ *            ispa_quantize_q_e4m3)
+ *   k8_cur : uint8 [n_q][H][128] codes, k_cur_scale fp32 [H] (e.g. the ring's)
+ *   k_ring_scale : the ring's key scales (as given to ispa_kv_append_qk8)
+ *   v_cur : bf16 [n_q][H][128]; out, lse, scale as in ispa_attn_full.
+ * Scale arrays live in device memory.  Errors as ispa_attn_full; a bf16 ring
+ * (or an e4m3 ring given to the bf16 entry points) is ISPA_ERR_INVALID_ARG. */
+ISPA_API ispa_status ispa_attn_full_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, const void* q8,
+                                        const float* q_scale, const void* k8_cur, const float* k_cur_scale,
+                                        const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
+                                        ispa_stream stream);
+ISPA_API ispa_status ispa_attn_local_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, ispa_window win,
+                                         const void* q8, const float* q_scale, const void* k8_cur,
+                                         const float* k_cur_scale, const void* v_cur, int32_t n_q, float scale,
+                                         void* out, float* lse, ispa_stream stream);
 
 /* ------------------------------------------------------------ W8A8 projection */
 /*

@@ -23,8 +23,9 @@ Linear: y[t, n] = a_scale[t] * w_scale[n] * sum_k dec(a_q[t, k]) * dec(w_q[n, k]
 
 8-bit query/key attention (SageAttention's 8-bit Q K^T with 16-bit P V, cited in Sec. 3.4):
 one scale per head, scale = fl32(amax / 448) over all the group's tokens (or a given scale, for
-keys appended into a cache), code = e4m3(fl32(x / scale)); the attention is then the plain
-attention of the dequantised q and k (codes times scale) with the unquantised v.
+keys appended into a cache), code = e4m3(fl32(x * fl32(1 / scale))); queries take one scale
+per head and block of 128 tokens (SageAttention's per-block granularity).  The attention is then
+the plain attention of the dequantised q and k (codes times scale) with the unquantised v.
 """
 from __future__ import annotations
 
@@ -111,10 +112,10 @@ def linear_w8a8(a_q, a_scale, w_q, w_scale) -> np.ndarray:
 
 
 def quantize_heads_with_scale(x, scale) -> np.ndarray:
-    """Token-major [n][H][d] values and per-head scales [H] -> codes e4m3(fl32(x / scale_h))."""
+    """Token-major [n][H][d] values and per-head scales [H] -> codes e4m3(fl32(x * fl32(1 / scale_h)))."""
     x = np.asarray(x, dtype=np.float32)
-    s = np.asarray(scale, dtype=np.float32)[None, :, None]
-    return encode((x / s).astype(np.float32))
+    inv = (np.float32(1) / np.asarray(scale, dtype=np.float32)).astype(np.float32)[None, :, None]
+    return encode((x * inv).astype(np.float32))
 
 
 def head_scales(x) -> np.ndarray:
@@ -133,4 +134,28 @@ def quantize_heads(x):
 def dequantize_heads(q, scale) -> np.ndarray:
     """codes [n][H][d], scales [H] -> float64 values."""
     return decode(q) * np.asarray(scale, np.float64)[None, :, None]
+
+
+def quantize_query_blocks(x, block: int = 128):
+    """Queries [n][H][d] -> (codes, scales [H][ceil(n / block)]): one scale per head and block of
+    `block` consecutive tokens, scale = fl32(amax / 448) (1 for an all-zero block)."""
+    x = np.asarray(x, dtype=np.float32)
+    n, H, _ = x.shape
+    nb = (n + block - 1) // block
+    scales = np.ones((H, nb), dtype=np.float32)
+    codes = np.zeros(x.shape, dtype=np.uint8)
+    for b in range(nb):
+        xb = x[b * block:(b + 1) * block]
+        s = head_scales(xb)
+        scales[:, b] = s
+        codes[b * block:(b + 1) * block] = quantize_heads_with_scale(xb, s)
+    return codes, scales
+
+
+def dequantize_query_blocks(q, scales, block: int = 128) -> np.ndarray:
+    q = np.asarray(q)
+    out = decode(q)
+    for b in range(scales.shape[1]):
+        out[b * block:(b + 1) * block] *= np.asarray(scales[:, b], np.float64)[None, :, None]
+    return out
 

@@ -25,12 +25,14 @@ ISPA_ERR_TIMEOUT = 5
 ISPA_ERR_CUDA = 6
 ISPA_ERR_WORKSPACE = 7
 ISPA_ATTN_FRAME_CAUSAL = 1   # option bit of the *_ex attention entry points
+ISPA_KV_BF16 = 0             # ring k_format values
+ISPA_KV_K_E4M3 = 1
 MAX_RANGES = 4
 
 
 class KVRing(Structure):
     _fields_ = [("num_heads", c_int32), ("head_dim", c_int32), ("tokens_per_frame", c_int32),
-                ("capacity_frames", c_int32), ("n_sink_frames", c_int32), ("reserved", c_int32),
+                ("capacity_frames", c_int32), ("n_sink_frames", c_int32), ("k_format", c_int32),
                 ("frames_written", c_int64), ("k", c_void_p), ("v", c_void_p)]
 
 
@@ -110,6 +112,14 @@ _SIGS = {
     "ispa_ls_accumulate": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
                                      c_void_p]),
     "ispa_ls_solve_workspace_size": (c_size_t, [c_int32, c_int32]),
+    "ispa_quantize_heads_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_quantize_q_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_quantize_k_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_kv_append_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
+    "ispa_attn_full_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                     c_int32, c_float, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_local_qk8": (c_int32, [POINTER(KVRing), c_void_p, Window, c_void_p, c_void_p, c_void_p, c_void_p,
+                                      c_void_p, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
     "ispa_quantize_rows_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_quantize_weight_e4m3": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_linear_w8a8": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_int32, c_int32, c_void_p,
@@ -343,4 +353,39 @@ def ispa_quantize_weight_e4m3(W, dW, D: int, D_out: int, q_t, scale, stream=None
 def ispa_linear_w8a8(a_q, a_scale, w_q, w_scale, T: int, D: int, D_out: int, out, stream=None) -> None:
     _check(lib().ispa_linear_w8a8(_ptr(a_q), _ptr(a_scale), _ptr(w_q), _ptr(w_scale), T, D, D_out, _ptr(out),
                                   _stream(stream)), "ispa_linear_w8a8")
+
+
+# ---------------------------------------------------------------- 8-bit Q K^T attention
+def ispa_quantize_heads_e4m3(x, n: int, H: int, d: int, q, scale, stream=None) -> None:
+    _check(lib().ispa_quantize_heads_e4m3(_ptr(x), n, H, d, _ptr(q), _ptr(scale), _stream(stream)),
+           "ispa_quantize_heads_e4m3")
+
+
+def ispa_kv_append_qk8(ring: KVRing, k_new, v_new, n_frames: int, k_scale, stream=None) -> None:
+    _check(lib().ispa_kv_append_qk8(ctypes.byref(ring), _ptr(k_new), _ptr(v_new), n_frames, _ptr(k_scale),
+                                    _stream(stream)), "ispa_kv_append_qk8")
+
+
+def ispa_attn_full_qk8(ring: KVRing, k_ring_scale, q8, q_scale, k8_cur, k_cur_scale, v_cur, n_q: int,
+                       scale: float, out, lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_full_qk8(ctypes.byref(ring), _ptr(k_ring_scale), _ptr(q8), _ptr(q_scale), _ptr(k8_cur),
+                                    _ptr(k_cur_scale), _ptr(v_cur), n_q, scale, _ptr(out), _ptr(lse),
+                                    _stream(stream)), "ispa_attn_full_qk8")
+
+
+def ispa_attn_local_qk8(ring: KVRing, k_ring_scale, win: Window, q8, q_scale, k8_cur, k_cur_scale, v_cur,
+                        n_q: int, scale: float, out, lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_local_qk8(ctypes.byref(ring), _ptr(k_ring_scale), win, _ptr(q8), _ptr(q_scale),
+                                     _ptr(k8_cur), _ptr(k_cur_scale), _ptr(v_cur), n_q, scale, _ptr(out),
+                                     _ptr(lse), _stream(stream)), "ispa_attn_local_qk8")
+
+
+def ispa_quantize_q_e4m3(x, n: int, H: int, d: int, q, scale, stream=None) -> None:
+    _check(lib().ispa_quantize_q_e4m3(_ptr(x), n, H, d, _ptr(q), _ptr(scale), _stream(stream)),
+           "ispa_quantize_q_e4m3")
+
+
+def ispa_quantize_k_e4m3(x, n: int, H: int, d: int, scale, q, stream=None) -> None:
+    _check(lib().ispa_quantize_k_e4m3(_ptr(x), n, H, d, _ptr(scale), _ptr(q), _stream(stream)),
+           "ispa_quantize_k_e4m3")
 

@@ -96,14 +96,14 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, 
 }
 
 bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], const uint64_t strides3[3],
-                    const uint32_t box4[4]) {
+                    const uint32_t box4[4], bool u8) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[4] = {dims4[0], dims4[1], dims4[2], dims4[3]};
   cuuint64_t strides[3] = {strides3[0], strides3[1], strides3[2]};
   cuuint32_t box[4] = {box4[0], box4[1], box4[2], box4[3]};
   cuuint32_t estr[4] = {1, 1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+  return fn(m, u8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -143,6 +143,8 @@ ispa_status check_ring(const ispa_kv_ring* r) {
       r->n_sink_frames < 0 || r->n_sink_frames >= r->capacity_frames || r->frames_written < 0)
     return ISPA_ERR_INVALID_ARG;
   if (r->head_dim != 64 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
+  if (r->k_format != ISPA_KV_BF16 && r->k_format != ISPA_KV_K_E4M3) return ISPA_ERR_INVALID_ARG;
+  if (r->k_format == ISPA_KV_K_E4M3 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
   if (static_cast<int64_t>(r->capacity_frames) * r->tokens_per_frame > INT32_MAX)
     return ISPA_ERR_INVALID_ARG;
   return ISPA_OK;
@@ -221,12 +223,21 @@ int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
   return tiles;
 }
 
+// 8-bit Q K^T: per-head e4m3 code scales of q, of the chunk keys and of the ring keys.
+struct Qk8Scales {
+  const float* q;
+  const float* k_cur;
+  const float* k_ring;
+};
+
 ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, const void* q,
                         const void* k_cur, const void* v_cur, int32_t n_q, float scale, uint32_t flags,
                         void* out, void* out_loc, float* lse, float* lse_loc, float* disc_part,
-                        cudaStream_t stream) {
+                        cudaStream_t stream, const Qk8Scales* qk8 = nullptr) {
   ispa_status st = check_ring(ring);
   if (st != ISPA_OK) return st;
+  if ((ring->k_format == ISPA_KV_K_E4M3) != (qk8 != nullptr)) return ISPA_ERR_INVALID_ARG;
+  if (qk8 && (!qk8->q || !qk8->k_cur || !qk8->k_ring)) return ISPA_ERR_INVALID_ARG;
   if (flags & ~static_cast<uint32_t>(ISPA_ATTN_FRAME_CAUSAL)) return ISPA_ERR_INVALID_ARG;
   if ((flags & ISPA_ATTN_FRAME_CAUSAL) && n_q % ring->tokens_per_frame != 0) return ISPA_ERR_INVALID_ARG;
   if (n_q <= 0 || !aligned16(q) || !aligned16(k_cur) || !aligned16(v_cur) || !aligned16(out) ||
@@ -300,9 +311,26 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const uint32_t box_q[4] = {64, static_cast<uint32_t>(kAttnBM), nb, 1};
   const uint32_t box_k[4] = {64, static_cast<uint32_t>(kAttnBN), nb, 1};
   CUtensorMap tq, tkr, tvr, tkc, tvc;
-  bool ok = encode_tmap_4d(&tq, q, dims_c, str_c, box_q) && encode_tmap_4d(&tkc, k_cur, dims_c, str_c, box_k) &&
-            encode_tmap_4d(&tvc, v_cur, dims_c, str_c, box_k) && encode_tmap_4d(&tkr, ring->k, dims_r, str_r, box_k) &&
-            encode_tmap_4d(&tvr, ring->v, dims_r, str_r, box_k);
+  bool ok = encode_tmap_4d(&tvc, v_cur, dims_c, str_c, box_k) && encode_tmap_4d(&tvr, ring->v, dims_r, str_r, box_k);
+  if (qk8) {
+    // e4m3 Q and K: a token's 128 features are one 128-byte row, so the column-block
+    // dimension has extent 1
+    const uint64_t dims_c8[4] = {128, static_cast<uint64_t>(n_q), 1, static_cast<uint64_t>(H)};
+    const uint64_t str_c8[3] = {128ull * H, 128, 128};
+    const uint64_t dims_r8[4] = {128, ring_tok, 1, static_cast<uint64_t>(H)};
+    const uint64_t str_r8[3] = {128, 128, 128 * ring_tok};
+    const uint32_t box_q8[4] = {128, static_cast<uint32_t>(kAttnBM), 1, 1};
+    const uint32_t box_k8[4] = {128, static_cast<uint32_t>(kAttnBN), 1, 1};
+    ok = ok && encode_tmap_4d(&tq, q, dims_c8, str_c8, box_q8, true) &&
+         encode_tmap_4d(&tkc, k_cur, dims_c8, str_c8, box_k8, true) &&
+         encode_tmap_4d(&tkr, ring->k, dims_r8, str_r8, box_k8, true);
+    p.q_scale = qk8->q;
+    p.kc_scale = qk8->k_cur;
+    p.kr_scale = qk8->k_ring;
+  } else {
+    ok = ok && encode_tmap_4d(&tq, q, dims_c, str_c, box_q) && encode_tmap_4d(&tkc, k_cur, dims_c, str_c, box_k) &&
+         encode_tmap_4d(&tkr, ring->k, dims_r, str_r, box_k);
+  }
   if (!ok) return ISPA_ERR_CUDA;
   if (launch_attention(HD, &tq, &tkr, &tvr, &tkc, &tvc, p, stream) != cudaSuccess) return ISPA_ERR_CUDA;
   return ISPA_OK;
@@ -392,7 +420,8 @@ ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream) {
 size_t ispa_ring_bytes(const ispa_kv_ring* r) {
   if (!r || r->num_heads <= 0 || r->head_dim <= 0 || r->tokens_per_frame <= 0 || r->capacity_frames <= 0)
     return 0;
-  return 2ull * r->num_heads * r->capacity_frames * r->tokens_per_frame * r->head_dim * 2ull;
+  const uint64_t elems = 1ull * r->num_heads * r->capacity_frames * r->tokens_per_frame * r->head_dim;
+  return elems * (r->k_format == ISPA_KV_K_E4M3 ? 1ull : 2ull) + elems * 2ull;
 }
 
 int32_t ispa_ring_slot(const ispa_kv_ring* r, int64_t frame) {
@@ -417,6 +446,7 @@ ispa_status ispa_kv_append_layers(ispa_kv_ring* rings, int32_t n_layers, const v
     const ispa_status st = check_ring(&rings[l]);
     if (st != ISPA_OK) return st;
     const ispa_kv_ring& r = rings[l];
+    if (r.k_format != ISPA_KV_BF16) return ISPA_ERR_INVALID_ARG;   // e4m3 keys: ispa_kv_append_qk8
     if (r.num_heads != r0.num_heads || r.head_dim != r0.head_dim || r.tokens_per_frame != r0.tokens_per_frame)
       return ISPA_ERR_INVALID_ARG;
     if (!aligned16(r.k) || !aligned16(r.v) || !aligned16(k_new[l]) || !aligned16(v_new[l]))
@@ -603,5 +633,69 @@ ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uin
   return ISPA_OK;
 }
 
+
+// ------------------------------------------------------------ 8-bit Q K^T attention
+
+ispa_status ispa_quantize_heads_e4m3(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q, float* scale,
+                                     ispa_stream stream) {
+  if (!x || !q || !scale || n <= 0 || H <= 0 || d <= 0 || !aligned16(x) || !aligned16(q))
+    return ISPA_ERR_INVALID_ARG;
+  if (d % 16 != 0 || H > 256) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_heads(x, n, H, d, q, scale, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_quantize_q_e4m3(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q, float* scale,
+                                 ispa_stream stream) {
+  if (!x || !q || !scale || n <= 0 || H <= 0 || d <= 0 || !aligned16(x) || !aligned16(q))
+    return ISPA_ERR_INVALID_ARG;
+  if (d % 16 != 0 || d > 256 || H > 65535) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_q_blocks(x, n, H, d, q, scale, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_quantize_k_e4m3(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* q,
+                                 ispa_stream stream) {
+  if (!x || !q || !scale || n <= 0 || H <= 0 || d <= 0 || !aligned16(x) || !aligned16(q))
+    return ISPA_ERR_INVALID_ARG;
+  if (d % 16 != 0) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_given(x, n, H, d, scale, q, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_kv_append_qk8(ispa_kv_ring* ring, const void* k_new, const void* v_new, int32_t n_frames,
+                               const float* k_scale, ispa_stream stream) {
+  const ispa_status st = check_ring(ring);
+  if (st != ISPA_OK) return st;
+  if (ring->k_format != ISPA_KV_K_E4M3 || !k_new || !v_new || !k_scale || n_frames <= 0) return ISPA_ERR_INVALID_ARG;
+  if (!aligned16(ring->k) || !aligned16(ring->v) || !aligned16(k_new) || !aligned16(v_new))
+    return ISPA_ERR_INVALID_ARG;
+  if (n_frames > kMaxAppendFrames || n_frames > ring->capacity_frames - ring->n_sink_frames) return ISPA_ERR_CAPACITY;
+  int32_t slots[kMaxAppendFrames];
+  for (int i = 0; i < n_frames; ++i) slots[i] = slot_of(ring, ring->frames_written + i);
+  const int64_t ring_tok = static_cast<int64_t>(ring->capacity_frames) * ring->tokens_per_frame;
+  if (launch_append_qk8(slots, n_frames, ring->tokens_per_frame, ring->num_heads, ring->head_dim, ring_tok, k_new,
+                        v_new, ring->k, ring->v, k_scale, stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  ring->frames_written += n_frames;
+  return ISPA_OK;
+}
+
+ispa_status ispa_attn_full_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, const void* q8,
+                               const float* q_scale, const void* k8_cur, const float* k_cur_scale, const void* v_cur,
+                               int32_t n_q, float scale, void* out, float* lse, ispa_stream stream) {
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale};
+  return attn_common(MODE_FULL, ring, ispa_window{0, 0}, q8, k8_cur, v_cur, n_q, scale, 0u, out, nullptr, lse,
+                     nullptr, nullptr, stream, &sc);
+}
+
+ispa_status ispa_attn_local_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, ispa_window win,
+                                const void* q8, const float* q_scale, const void* k8_cur, const float* k_cur_scale,
+                                const void* v_cur, int32_t n_q, float scale, void* out, float* lse,
+                                ispa_stream stream) {
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale};
+  return attn_common(MODE_LOCAL, ring, win, q8, k8_cur, v_cur, n_q, scale, 0u, out, nullptr, lse, nullptr, nullptr,
+                     stream, &sc);
+}
 
 }  // extern "C"

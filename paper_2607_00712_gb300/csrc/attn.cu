@@ -65,19 +65,23 @@ constexpr int HALF_COLS = BN / 2;          // score columns per softmax warp
 constexpr int P_HALF = HALF_COLS / 2;      // packed bf16 P columns per softmax warp
 static_assert(BN % 16 == 0 && BN <= 256 && HALF_COLS % 8 == 0 && P_HALF % 4 == 0, "key tile shape");
 
-template <int HD>
+// QK8: Q and K as e4m3 codes (one 128-byte swizzled row = the 128 features of a token), S by
+// kind::f8f6f4 UMMAs with K = 32; V, P and O as in the bf16 path.
+template <int HD, bool QK8 = false>
 struct Cfg {
-  static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per tile row
+  static_assert(!QK8 || HD == 128, "8-bit Q K^T is built for head_dim 128");
+  static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per bf16 tile row
   static constexpr int QBOX = BM * 128;         // [128 rows][64 bf16] = 16 KB
   static constexpr int KBOX = BN * 128;         // [176 rows][64 bf16] = 22 KB
-  static constexpr int Q_TILE = NBOX * QBOX;
-  static constexpr int KV_TILE = NBOX * KBOX;   // one K or V tile
-  static constexpr int KST = HD == 128 ? 2 : 4;  // K stages
-  static constexpr int VST = HD == 128 ? 2 : 4;  // V stages
+  static constexpr int Q_TILE = QK8 ? BM * HD : NBOX * QBOX;
+  static constexpr int K_TILE = QK8 ? BN * HD : NBOX * KBOX;
+  static constexpr int V_TILE = NBOX * KBOX;
+  static constexpr int KST = (HD == 128 && !QK8) ? 2 : 4;  // K stages
+  static constexpr int VST = HD == 128 ? 2 : 4;            // V stages
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = Q_TILE;
-  static constexpr int OFF_V = OFF_K + KST * KV_TILE;
-  static constexpr int OFF_X = OFF_V + VST * KV_TILE;          // exchange arrays (fp32)
+  static constexpr int OFF_V = OFF_K + KST * K_TILE;
+  static constexpr int OFF_X = OFF_V + VST * V_TILE;          // exchange arrays (fp32)
   static constexpr int X_FLOATS = 2 * 2 * BM;  // max[parity][half][BM]; the epilogue reuses it
   static constexpr int OFF_BAR = OFF_X + X_FLOATS * 4;
   static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
@@ -85,7 +89,7 @@ struct Cfg {
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
   static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
-  static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, false, false);
+  static constexpr uint32_t IDESC_QK = QK8 ? idesc_e4m3(BM, BN) : idesc_bf16(BM, BN, false, false);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, HD, false, true);
   static_assert(COL_O + HD <= 512, "TMEM columns");
   static_assert(KBOX % 1024 == 0 && QBOX % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
@@ -145,12 +149,12 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 
 }  // namespace
 
-template <int HD>
+template <int HD, bool QK8>
 __global__ void __launch_bounds__(NTHREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kr,
                 const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_kc,
                 const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
-  using C = Cfg<HD>;
+  using C = Cfg<HD, QK8>;
   // The dynamic shared window must start on a 1 KB boundary (the swizzle atoms of the
   // TMA boxes); the declaration asks for it and the check below enforces it.
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -241,8 +245,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const int row = p.seg[kseg].start + koff;
           const int ks = t % C::KST;
           if (!mbar_wait(b.k_empty0 + 8 * ks, ((t / C::KST) & 1) ^ 1, wc, 1, t)) break;
-          mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::KV_TILE);
-          const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
+          mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::K_TILE);
+          const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
           tma_load_4d(sK, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0, row, 0, head);
           nk = t + 1;
           trace_event(p.trace, p.trace_tiles, t, 6);
@@ -254,8 +258,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const int row = p.seg[vseg].start + voff;
           const int vs = j % C::VST;
           if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
-          mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::KV_TILE);
-          const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
+          mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::V_TILE);
+          const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
           tma_load_4d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0, row, 0, head);
           nv = j + 1;
           trace_event(p.trace, p.trace_tiles, j, 7);
@@ -281,13 +285,20 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int ks = j % C::KST;
         if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc, 4, j)) return false;
         tc_fence_after();
-        const uint32_t sK = sbase + C::OFF_K + ks * C::KV_TILE;
+        const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
         const uint32_t d = tmem + C::COL_S0 + (j & 1) * BN;
+        if constexpr (QK8) {
 #pragma unroll
-        for (int k = 0; k < HD / 16; ++k) {
-          const uint32_t kin = (k & 3) * 32;
-          umma_ss(d, sw128_desc(sQ + (k >> 2) * C::QBOX + kin, 16, 1024),
-                  sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
+          for (int k = 0; k < HD / 32; ++k)   // K = 32 codes per step inside the 128-byte row
+            umma_f8(d, sw128_desc(sQ + 32 * k, 16, 1024), sw128_desc(sK + 32 * k, 16, 1024), C::IDESC_QK,
+                    k > 0 ? 1u : 0u);
+        } else {
+#pragma unroll
+          for (int k = 0; k < HD / 16; ++k) {
+            const uint32_t kin = (k & 3) * 32;
+            umma_ss(d, sw128_desc(sQ + (k >> 2) * C::QBOX + kin, 16, 1024),
+                    sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
+          }
         }
         tc_commit(b.s_full0 + 8 * (j & 1));
         tc_commit(b.k_empty0 + 8 * ks);
@@ -301,7 +312,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         trace_event(p.trace, p.trace_tiles, j, 3);
         if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
         tc_fence_after();
-        const uint32_t sV = sbase + C::OFF_V + vs * C::KV_TILE;
+        const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
         const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
 #pragma unroll
         for (int k = 0; k < BN / 16; ++k) {
@@ -328,8 +339,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const bool row_ok = qrow < p.n_q;
     const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int D = p.num_heads * HD;
-    const float sl2 = p.scale_log2;
-    const uint64_t sl2x2 = f2_pack(sl2, sl2);
+    // log2-domain score scale; with 8-bit Q and K it also carries the per-head code scales,
+    // which differ between ring keys and chunk keys
+    float sl2_ring = p.scale_log2, sl2_chunk = p.scale_log2;
+    if constexpr (QK8) {
+      const float qs = p.q_scale[static_cast<int64_t>(head) * gridDim.x + q_tile];   // [H][query blocks]
+      sl2_ring = p.scale_log2 * qs * p.kr_scale[head];
+      sl2_chunk = p.scale_log2 * qs * p.kc_scale[head];
+    }
     float m_run = -INFINITY, l_run = 0.f;  // l_run: this warp's column half only
     int seg = 0, off = 0;
     bool ok = true;
@@ -402,6 +419,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
       if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 0);
       const int valid = min(BN, p.seg[seg].count - off);
+      const float sl2 = p.seg[seg].src != 0 ? sl2_chunk : sl2_ring;
+      const uint64_t sl2x2 = f2_pack(sl2, sl2);
       uint32_t s[HALF_COLS];
       float mx = -INFINITY;
       if (ok) {
@@ -511,29 +530,33 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
 }
 
-template <int HD>
+template <int HD, bool QK8>
 static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, const CUtensorMap* tvr,
                              const CUtensorMap* tkc, const CUtensorMap* tvc, const AttnParams& p,
                              cudaStream_t s) {
-  using C = Cfg<HD>;
+  using C = Cfg<HD, QK8>;
   static bool attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, QK8>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_done[dev] = true;
   }
   dim3 grid((p.n_q + BM - 1) / BM, p.num_heads);
-  attn_kernel<HD><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
+  attn_kernel<HD, QK8><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
   return cudaGetLastError();
 }
 
 cudaError_t launch_attention(int head_dim, const CUtensorMap* tq, const CUtensorMap* tkr,
                              const CUtensorMap* tvr, const CUtensorMap* tkc,
                              const CUtensorMap* tvc, const AttnParams& p, cudaStream_t s) {
-  if (head_dim == 128) return launch_hd<128>(tq, tkr, tvr, tkc, tvc, p, s);
-  if (head_dim == 64) return launch_hd<64>(tq, tkr, tvr, tkc, tvc, p, s);
+  if (p.q_scale) {
+    if (head_dim == 128) return launch_hd<128, true>(tq, tkr, tvr, tkc, tvc, p, s);
+    return cudaErrorInvalidValue;
+  }
+  if (head_dim == 128) return launch_hd<128, false>(tq, tkr, tvr, tkc, tvc, p, s);
+  if (head_dim == 64) return launch_hd<64, false>(tq, tkr, tvr, tkc, tvc, p, s);
   return cudaErrorInvalidValue;
 }
 

@@ -47,6 +47,10 @@ struct AttnParams {
   uint64_t* trace;         // debug per-tile cycle trace of CTA (0,0) or null: [tile][8]
   int32_t trace_tiles;
   int32_t pad2;
+  // 8-bit Q K^T (null for bf16 Q and K): per-head e4m3 code scales of q, chunk keys, ring keys
+  const float* q_scale;
+  const float* kc_scale;
+  const float* kr_scale;
 };
 
 // Launch the attention kernel.  tensor maps are encoded by the caller.
@@ -100,14 +104,25 @@ cudaError_t launch_w8a8_gemm(const uint8_t* a_q, const float* a_scale, const uin
                              int32_t T, int32_t D, int32_t Dout, void* out, int* status, uint64_t wait_limit_ns,
                              cudaStream_t s);
 
+// ------------------------------------------------------------ 8-bit Q K^T
+cudaError_t launch_quant_heads(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q, float* scale,
+                               cudaStream_t s);
+cudaError_t launch_quant_q_blocks(const void* x, int64_t n, int32_t H, int32_t d, uint8_t* q, float* scale,
+                                  cudaStream_t s);
+cudaError_t launch_quant_given(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* q,
+                               cudaStream_t s);
+cudaError_t launch_append_qk8(const int32_t* slots, int32_t n_frames, int32_t P, int32_t H, int32_t d,
+                              int64_t ring_tok, const void* k_src, const void* v_src, void* k_dst, void* v_dst,
+                              const float* k_scale, cudaStream_t s);
+
 // ------------------------------------------------------------ misc
 int* device_status_ptr();  // library status word on the current device (nullptr on error)
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                     uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                     uint32_t b2);
-// bf16, 128-byte swizzle, rank 4 (dims / strides in bytes for dims 1-3 / box).
+// 128-byte swizzle, rank 4 (dims / strides in bytes for dims 1-3 / box).
 bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], const uint64_t strides3[3],
-                    const uint32_t box4[4]);
+                    const uint32_t box4[4], bool u8 = false);   // u8: uint8 elements instead of bf16
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
 // uint8 elements, 128-byte swizzle, rank 2.

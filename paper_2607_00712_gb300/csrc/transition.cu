@@ -172,6 +172,7 @@ ispa_status ispa_apply_absorption_bf16(void* W, const float* dW, int32_t dim, in
 ispa_status ispa_ring_compact(const ispa_kv_ring* src, ispa_window win, ispa_kv_ring* dst, ispa_stream stream) {
   if (!src || !dst || win.n_sink_frames < 0 || win.n_recent_frames < 0) return ISPA_ERR_INVALID_ARG;
   if (ispa_ring_bytes(src) == 0 || ispa_ring_bytes(dst) == 0) return ISPA_ERR_INVALID_ARG;
+  if (src->k_format != ISPA_KV_BF16 || dst->k_format != ISPA_KV_BF16) return ISPA_ERR_UNSUPPORTED;
   if (src->num_heads != dst->num_heads || src->head_dim != dst->head_dim ||
       src->tokens_per_frame != dst->tokens_per_frame || dst->n_sink_frames != win.n_sink_frames ||
       dst->capacity_frames != win.n_sink_frames + win.n_recent_frames || win.n_recent_frames < 1)

@@ -155,21 +155,6 @@ constexpr int QK = 128;        // K (bytes = codes) per stage: one 128-byte swiz
 constexpr int Q_THREADS = 192;
 constexpr uint64_t Q_DRAIN_NS = 200ull * 1000 * 1000;
 
-__host__ __device__ constexpr uint32_t idesc_e4m3(int M, int N) {
-  // D fp32 (bit 4); A and B e4m3 (format 0), both K-major; N >> 3 at bit 17, M >> 4 at bit 24
-  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
-}
-
-__device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                        uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
 template <int BN>
 struct QCfg {
   // 256-column tiles: 4 stages, one CTA per SM; 128-column tiles: 3 stages (96 KB) so that two

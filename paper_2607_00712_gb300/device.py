@@ -19,15 +19,17 @@ def to_f32(t: torch.Tensor) -> np.ndarray:
 
 
 class Ring:
-    """A caller-owned KV ring: two bf16 [H][cap*P][d] tensors plus the C struct."""
+    """A caller-owned KV ring: K and V [H][cap*P][d] tensors plus the C struct.
+
+    k_e4m3: keys as e4m3 codes (uint8), for the 8-bit query/key attention entry points."""
 
     def __init__(self, num_heads: int, head_dim: int, tokens_per_frame: int, capacity_frames: int,
-                 n_sink_frames: int = 0, device="cuda"):
+                 n_sink_frames: int = 0, device="cuda", k_e4m3: bool = False):
         shape = (num_heads, capacity_frames * tokens_per_frame, head_dim)
-        self.k = torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        self.k = torch.zeros(shape, dtype=torch.uint8 if k_e4m3 else torch.bfloat16, device=device)
         self.v = torch.zeros(shape, dtype=torch.bfloat16, device=device)
-        self.c = KVRing(num_heads, head_dim, tokens_per_frame, capacity_frames, n_sink_frames, 0, 0,
-                        self.k.data_ptr(), self.v.data_ptr())
+        self.c = KVRing(num_heads, head_dim, tokens_per_frame, capacity_frames, n_sink_frames, 1 if k_e4m3 else 0,
+                        0, self.k.data_ptr(), self.v.data_ptr())
 
     @property
     def frames_written(self) -> int:

@@ -143,3 +143,15 @@ def test_quantize_with_scale_saturates_outliers():
     x = np.array([[[1.0, -2.0, 1000.0, -1e6]]], dtype=np.float32)
     q = qt.quantize_heads_with_scale(x, np.array([1.0], np.float32))
     assert list(qt.decode(q).ravel()) == [1.0, -2.0, 448.0, -448.0]
+
+
+def test_query_blocks_are_per_head_quantisation_of_each_block():
+    r = np.random.default_rng(7)
+    x = (r.standard_normal((300, 2, 8)) * r.uniform(0.1, 9, (300, 1, 1))).astype(np.float32)
+    q, s = qt.quantize_query_blocks(x, block=128)
+    assert s.shape == (2, 3)
+    for b in range(3):
+        qb, sb = qt.quantize_heads(x[b * 128:(b + 1) * 128])
+        assert np.array_equal(q[b * 128:(b + 1) * 128], qb) and np.array_equal(s[:, b], sb)
+    back = qt.dequantize_query_blocks(q, s)
+    assert np.all(np.abs(back - x) <= 2.0 ** -4 * np.abs(x) * (1 + 1e-6) + 2.0 ** -10 * s.max())
