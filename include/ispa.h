@@ -468,6 +468,14 @@ ISPA_API ispa_status ispa_attn_local_qk8(const ispa_kv_ring* ring, const float* 
                                          const void* q8, const float* q_scale, const void* k8_cur,
                                          const float* k_cur_scale, const void* v_cur, int32_t n_q, float scale,
                                          void* out, float* lse, ispa_stream stream);
+/* ispa_attn_dual over a ring with e4m3 keys (scales as above; other arguments
+ * and the workspace as in ispa_attn_dual). */
+ISPA_API ispa_status ispa_attn_dual_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, ispa_window win,
+                                        const void* q8, const float* q_scale, const void* k8_cur,
+                                        const float* k_cur_scale, const void* v_cur, int32_t n_q, float scale,
+                                        void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                                        float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                                        ispa_stream stream);
 
 /* ------------------------------------------------------------ W8A8 projection */
 /*

@@ -118,6 +118,9 @@ _SIGS = {
     "ispa_kv_append_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
     "ispa_attn_full_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                      c_int32, c_float, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_dual_qk8": (c_int32, [POINTER(KVRing), c_void_p, Window, c_void_p, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_int32, c_float, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_void_p, c_size_t, c_void_p]),
     "ispa_attn_local_qk8": (c_int32, [POINTER(KVRing), c_void_p, Window, c_void_p, c_void_p, c_void_p, c_void_p,
                                       c_void_p, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
     "ispa_quantize_rows_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_void_p, c_void_p, c_void_p]),
@@ -388,4 +391,13 @@ def ispa_quantize_q_e4m3(x, n: int, H: int, d: int, q, scale, stream=None) -> No
 def ispa_quantize_k_e4m3(x, n: int, H: int, d: int, scale, q, stream=None) -> None:
     _check(lib().ispa_quantize_k_e4m3(_ptr(x), n, H, d, _ptr(scale), _ptr(q), _stream(stream)),
            "ispa_quantize_k_e4m3")
+
+
+def ispa_attn_dual_qk8(ring: KVRing, k_ring_scale, win: Window, q8, q_scale, k8_cur, k_cur_scale, v_cur, n_q: int,
+                       scale: float, a_full, a_loc, disc, disc_sq_sum, lse_full=None, lse_loc=None, workspace=None,
+                       ws_bytes: int = 0, stream=None) -> None:
+    _check(lib().ispa_attn_dual_qk8(ctypes.byref(ring), _ptr(k_ring_scale), win, _ptr(q8), _ptr(q_scale),
+                                    _ptr(k8_cur), _ptr(k_cur_scale), _ptr(v_cur), n_q, scale, _ptr(a_full),
+                                    _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full), _ptr(lse_loc),
+                                    _ptr(workspace), ws_bytes, _stream(stream)), "ispa_attn_dual_qk8")
 

@@ -689,6 +689,24 @@ ispa_status ispa_attn_full_qk8(const ispa_kv_ring* ring, const float* k_ring_sca
                      nullptr, nullptr, stream, &sc);
 }
 
+ispa_status ispa_attn_dual_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, ispa_window win, const void* q8,
+                               const float* q_scale, const void* k8_cur, const float* k_cur_scale, const void* v_cur,
+                               int32_t n_q, float scale, void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                               float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes, ispa_stream stream) {
+  if (!ring || !disc || !disc_sq_sum) return ISPA_ERR_INVALID_ARG;
+  const size_t need = ispa_attn_dual_workspace_size(ring->num_heads, n_q);
+  if (need == 0) return ISPA_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
+  float* part = static_cast<float*>(workspace);
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale};
+  const ispa_status st = attn_common(MODE_DUAL, ring, win, q8, k8_cur, v_cur, n_q, scale, 0u, a_full, a_loc,
+                                     lse_full, lse_loc, part, stream, &sc);
+  if (st != ISPA_OK) return st;
+  if (launch_disc_reduce(part, ring->num_heads, n_q, disc, disc_sq_sum, stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
 ispa_status ispa_attn_local_qk8(const ispa_kv_ring* ring, const float* k_ring_scale, ispa_window win,
                                 const void* q8, const float* q_scale, const void* k8_cur, const float* k_cur_scale,
                                 const void* v_cur, int32_t n_q, float scale, void* out, float* lse,

@@ -164,6 +164,26 @@ def test_qk8_attention_ragged_and_wrapped():
         assert np.abs(l - rl).max() < 2e-3
 
 
+def test_qk8_dual_matches_oracle():
+    st = Qk8Step(28, P=100, H=3, n_past=9, n_chunk_frames=3, capacity=8, n_sink_pinned=1)
+    D = st.H * st.d
+    a_full = torch.empty(st.n_q, D, dtype=torch.bfloat16, device="cuda")
+    a_loc = torch.empty_like(a_full)
+    disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    wsb = abi.ispa_attn_dual_workspace_size(st.H, st.n_q)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    abi.ispa_attn_dual_qk8(st.ring.c, st.k_ring_scale, Window(1, 2), st.q8, st.q_scale, st.k8c, st.kc_scale, st.vc,
+                           st.n_q, 0.0, a_full, a_loc, disc, dsum, None, None, ws, wsb)
+    torch.cuda.synchronize()
+    r = at.attn_dual(*st.args, 1, 2)
+    assert_close_attn(to_f32(a_full).reshape(r["a_full"].shape), r["a_full"], "qk8 dual full")
+    assert_close_attn(to_f32(a_loc).reshape(r["a_loc"].shape), r["a_loc"], "qk8 dual loc")
+    got = to_f32(disc)
+    own = np.sqrt(((to_f32(a_full).astype(np.float64) - to_f32(a_loc)) ** 2).sum(1))
+    assert np.allclose(got, own, rtol=1e-5, atol=1e-6)
+
+
 def test_qk8_saturated_ring_keys_still_match_their_dequantised_values():
     # ring scales deliberately too small: the largest keys saturate at +-448 codes, and the
     # attention is that of the saturated (dequantised) keys
