@@ -25,6 +25,11 @@
  *   - Kernels never spin without bound: a wait that runs out records a device
  *     error, which ispa_last_device_error() reports as ISPA_ERR_TIMEOUT.
  *   - Head dims supported: 64 and 128.  Tokens per frame P >= 1.
+ *   - Threads: entry points may be called from several host threads for
+ *     different rings, states and streams.  ispa_set_wait_limit_ns and the
+ *     ispa_debug_* setters change process-wide settings without locking; set
+ *     them before work is issued from other threads.  The device error record
+ *     is one per device and shared by every call on it.
  */
 #ifndef ISPA_H_
 #define ISPA_H_

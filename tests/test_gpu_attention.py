@@ -212,3 +212,12 @@ def test_back_to_back_calls_without_host_sync():
     assert np.array_equal(to_f32(outs[1]).reshape(l_ref.shape), l_ref)
     assert np.array_equal(to_f32(outs[2]).reshape(o_ref.shape), g_ref["a_full"])
     assert np.array_equal(to_f32(outs[3]).reshape(o_ref.shape), g_ref["a_loc"])
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_minimum_sizes_one_query_one_head(d):
+    # n_q = 1 (one query of a one-token chunk frame), one head, one-token frames: the
+    # smallest step the boundary accepts
+    st = Step(51, P=1, H=1, d=d, n_past=5, n_chunk_frames=1, capacity=3, n_sink_pinned=1)
+    assert st.n_q == 1
+    _check_all_modes(st, (1, 1))
