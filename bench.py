@@ -14,6 +14,12 @@ value = attention FLOPs of the three modes (4*Nq*Nk*d*H each) / device time of t
 L2 is flushed (256 MB write) between timed steps, outside the timed events.
 Inputs are synthetic (seeded N(0,1) q/k/v with per-frame key offsets), bf16.
 
+The "extras" object also times, outside the step: the two-call dual decomposition, the
+solve, the W8A8 projection, the 8-bit Q K^T attention, and (unless --no-configs) the 20-step
+AR rollout of the whole layer stack (30 layers at 1.3B, 40 at 14B; half F-layers over a cache
+growing to 60 frames, half L-layers; batched append per step) and the warmup-to-transition
+path (8 dual steps on a 24-frame cache with LS accumulation, then one solve).
+
 Under torchrun (N > 1) every rank runs an independent replica on its own GPU
 (the path has no exchange step); timing is max over ranks and value sums ranks.
 --impl reference times the fp64 CPU oracle on a bounded sample of the same step.
@@ -43,6 +49,7 @@ MODELS = {
     "1.3b": (12, 128, 1560, 3, 18, 6),
     "14b": (40, 128, 1560, 3, 18, 6),
 }
+MODEL_LAYERS = {"1.3b": 30, "14b": 40}   # transformer blocks of the rollout workloads (half F, half L)
 
 
 def log(*a):
@@ -316,6 +323,10 @@ def run_ours(args, rank, world, local_rank):
     log(f"[bench] timed steps done at {time.perf_counter() - t_start:.1f} s")
     extras = run_extras(r, wl, device)
     log(f"[bench] extras done at {time.perf_counter() - t_start:.1f} s")
+    if args.configs:
+        extras["rollout"] = run_rollout(wl, device, MODEL_LAYERS[args.model])
+        extras["warmup_to_transition"] = run_warmup(wl, device)
+        log(f"[bench] rollout and warmup configs done at {time.perf_counter() - t_start:.1f} s")
     e2e = run_e2e(r, args, device, flops_step, world)
     log(f"[bench] e2e done at {time.perf_counter() - t_start:.1f} s")
 
@@ -492,6 +503,155 @@ def run_w8a8(r, wl, device, W, dW, reps):
                 w8a8_shape=f"{T} x {D} -> {D}")
 
 
+def _device_qkv(g, n_frames, P, H, d):
+    """One layer's chunk q, k, v drawn on the device with the synthetic recipe of the parity
+    inputs: N(0, 1) entries, every key of a frame and head shifted by an offset vector
+    ~ N(0, 0.5^2), rounded to bf16."""
+    import torch
+    dev = g.device
+    q = torch.randn(n_frames * P, H, d, device=dev, generator=g)
+    k = torch.randn(n_frames, P, H, d, device=dev, generator=g)
+    k += 0.5 * torch.randn(n_frames, 1, H, d, device=dev, generator=g)
+    v = torch.randn(n_frames * P, H, d, device=dev, generator=g)
+    return tuple(x.reshape(n_frames * P, H, d).to(torch.bfloat16) for x in (q, k, v))
+
+
+def run_rollout(wl, device, n_layers, steps=20):
+    """The AR rollout workload: `steps` chunk steps of `n_layers` blocks alternating F-layers
+    (attention over every past frame; the cache grows from 0 to 3 * (steps - 1) frames, up to
+    93,600 keys) and L-layers (chunk + 6-frame window), each step ending with the batched KV
+    append of all layers.  Every layer has its own ring and its own chunk q, k, v (drawn on the
+    device before each step, outside the timed events); L2 is not flushed between layers.
+    The rollout's keys (the F-rings hold up to 60 frames) keep the working set far above L2."""
+    import torch
+    from paper_2607_00712_gb300 import abi
+    from paper_2607_00712_gb300.device import Ring, Window
+    H, d, P, L, Wn, nq = (wl[k] for k in ("H", "d", "P", "L", "W", "nq"))
+    cap_f = L * steps
+    rings = [Ring(H, d, P, cap_f if li % 2 == 0 else Wn, 0, device) for li in range(n_layers)]
+    win = Window(0, Wn)
+    outs = torch.empty(nq, H * d, dtype=torch.bfloat16, device=device)
+    arr = (abi.KVRing * n_layers)()
+    s = torch.cuda.current_stream(device)
+    e0, ea, e1 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    g = torch.Generator(device=device)
+    g.manual_seed(7)
+    total_ms, append_ms, flops, step_ms = 0.0, 0.0, 0.0, []
+    for step in range(steps):
+        past = L * step
+        chunk = [_device_qkv(g, L, P, H, d) for _ in range(n_layers)]
+        torch.cuda.synchronize(device)
+        e0.record(s)
+        for li in range(n_layers):
+            q, kc, vc = chunk[li]
+            if li % 2 == 0:
+                abi.ispa_attn_full(rings[li].c, q, kc, vc, nq, 0.0, outs, None, s)
+                flops += attn_flops(nq, past * P + nq, d, H)
+            else:
+                abi.ispa_attn_local(rings[li].c, win, q, kc, vc, nq, 0.0, outs, None, s)
+                flops += attn_flops(nq, min(past, Wn) * P + nq, d, H)
+        for li in range(n_layers):
+            arr[li] = rings[li].c
+        ea.record(s)
+        abi.ispa_kv_append_layers(arr, [c[1] for c in chunk], [c[2] for c in chunk], L, s)
+        for li in range(n_layers):
+            rings[li].c.frames_written = arr[li].frames_written
+        e1.record(s)
+        torch.cuda.synchronize(device)
+        step_ms.append(e0.elapsed_time(e1))
+        total_ms += step_ms[-1]
+        append_ms += ea.elapsed_time(e1)
+        if step < steps - 1:
+            del chunk
+    # the append alone: one batched launch over all layers against one launch per layer
+    # (the rings are full here, so every append evicts the oldest frames)
+    app_bytes = n_layers * 2 * 2 * nq * H * d * 2
+    reps = 5
+    torch.cuda.synchronize(device)
+    e0.record(s)
+    for _ in range(reps):
+        for li in range(n_layers):
+            arr[li] = rings[li].c
+        abi.ispa_kv_append_layers(arr, [c[1] for c in chunk], [c[2] for c in chunk], L, s)
+        for li in range(n_layers):
+            rings[li].c.frames_written = arr[li].frames_written
+    e1.record(s)
+    torch.cuda.synchronize(device)
+    batched = e0.elapsed_time(e1) / reps
+    e0.record(s)
+    for _ in range(reps):
+        for li in range(n_layers):
+            abi.ispa_kv_append(rings[li].c, chunk[li][1], chunk[li][2], L, s)
+    e1.record(s)
+    torch.cuda.synchronize(device)
+    per_layer = e0.elapsed_time(e1) / reps
+    return dict(layers=n_layers, steps=steps, max_keys=(L * (steps - 1)) * P + nq, ms=round(total_ms, 2),
+                first_step_ms=round(step_ms[0], 3), last_step_ms=round(step_ms[-1], 3),
+                attention_tflop=round(flops / 1e12, 2),
+                attention_tflops=round(flops / ((total_ms - append_ms) * 1e-3) / 1e12, 1),
+                append_ms_per_step=round(append_ms / steps, 4),
+                append_all_layers=dict(batched_ms=round(batched, 4), per_layer_calls_ms=round(per_layer, 4),
+                                       batched_gbs=round(app_bytes / (batched * 1e-3) / 1e9, 0),
+                                       per_layer_gbs=round(app_bytes / (per_layer * 1e-3) / 1e9, 0)))
+
+
+def run_warmup(wl, device, steps=8, cache_frames=24):
+    """The warmup-to-transition workload: `steps` dual passes (full set = a 24-frame cache +
+    the chunk, local = chunk + 6-frame window) with the discrepancy reduction and the LS
+    accumulation of every step's A_loc / A_full, then the closed-form solve once."""
+    import torch
+    from paper_2607_00712_gb300 import abi, synth
+    from paper_2607_00712_gb300.device import LS, Ring, Window
+    H, d, P, L, Wn, nq, D = (wl[k] for k in ("H", "d", "P", "L", "W", "nq", "D"))
+    g = torch.Generator(device=device)
+    g.manual_seed(11)
+    ring = Ring(H, d, P, cache_frames, 0, device)
+    for f0 in range(0, cache_frames, L):
+        _, kk, vv = _device_qkv(g, L, P, H, d)
+        abi.ispa_kv_append(ring.c, kk, vv, L)
+    win = Window(0, Wn)
+    st = LS(D, device)
+    a_full = torch.empty(nq, D, dtype=torch.bfloat16, device=device)
+    a_loc = torch.empty_like(a_full)
+    disc = torch.empty(nq, dtype=torch.float32, device=device)
+    dsum = torch.zeros(1, dtype=torch.float32, device=device)
+    wsb = abi.ispa_attn_dual_workspace_size(H, nq)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=device)
+    lwsb = abi.ispa_ls_accumulate_workspace_size(D, nq)
+    lws = torch.empty(lwsb, dtype=torch.uint8, device=device)
+    qkv = [_device_qkv(g, L, P, H, d) for _ in range(steps)]
+    s = torch.cuda.current_stream(device)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    t_dual = t_ls = 0.0
+    torch.cuda.synchronize(device)
+    for q, kc, vc in qkv:
+        ev[0].record(s)
+        abi.ispa_attn_dual(ring.c, win, q, kc, vc, nq, 0.0, a_full, a_loc, disc, dsum, None, None, ws, wsb, s)
+        ev[1].record(s)
+        abi.ispa_ls_accumulate(st.c, a_loc, a_full, nq, lws, lwsb, s)
+        ev[2].record(s)
+        torch.cuda.synchronize(device)
+        t_dual += ev[0].elapsed_time(ev[1])
+        t_ls += ev[1].elapsed_time(ev[2])
+    W = torch.from_numpy(synth.make_weight(3, D, D)).to(device)
+    dW = torch.empty(D, D, dtype=torch.float32, device=device)
+    swsb = abi.ispa_ls_solve_workspace_size(D, D)
+    sws = torch.empty(swsb, dtype=torch.uint8, device=device)
+    torch.cuda.synchronize(device)
+    t0 = time.perf_counter()
+    nk = cache_frames * P + nq
+    out = dict(steps=steps, keys_full=nk, dual_ms_per_step=round(t_dual / steps, 4),
+               dual_tflops=round(attn_flops(nq, nk, d, H) / (t_dual / steps * 1e-3) / 1e12, 1),
+               ls_accumulate_ms_per_step=round(t_ls / steps, 4), tokens=steps * nq,
+               disc_sq_sum=float(dsum.item()))
+    try:
+        out["eps"] = abi.ispa_ls_solve(st.c, W, D, 1e-3, dW, sws, swsb, s)
+        out["solve_ms"] = round((time.perf_counter() - t0) * 1e3, 2)
+    except abi.IspaError as e:
+        out["solve_error"] = str(e)
+    return out
+
+
 def run_e2e(r, args, device, flops_step, world):
     """The same step through the C-ABI with pinned host inputs / outputs copied inside the timed region.
 
@@ -628,6 +788,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--model", choices=sorted(MODELS), default="1.3b")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--no-configs", dest="configs", action="store_false",
+                    help="skip the rollout and warmup-to-transition workloads in the extras")
     ap.add_argument("--cpu-sample-rows", type=int, default=1024)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--watchdog", type=float, default=300.0, help="dump Python stacks after this many s")
