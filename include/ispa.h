@@ -128,8 +128,10 @@ typedef struct {
  *   G = A_loc^T A_loc   rows [0,dim)     cols [0,dim)
  *   X = A_loc^T Delta   rows [0,dim)     cols [dim,2dim)
  *   S = Delta^T Delta   rows [dim,2dim)  cols [dim,2dim)
- * Only the upper 128x128 tiles of G and S (diagonal tiles in full) and all of
- * X are maintained; the rest of the buffer is left untouched.  The paper's
+ * All of X is maintained, and of G and S every 128x128 tile on or above the
+ * diagonal (tile (i, j), j >= i, diagonal tiles in full); with dim a multiple
+ * of 256 the tiles (2k+1, 2k) just below the diagonal hold their sums too.
+ * No other part of the buffer is written.  The paper's
  * A_loc^T R equals X W and is formed by the solve.  n_tokens counts the rows
  * accumulated (host side).  Plain data: copying it checkpoints the warmup.
  */
