@@ -12,12 +12,14 @@
 // oracle's): amax = max |x|; inv = 448 / amax, scale = amax / 448 (both 1 for an all-zero
 // group); code = e4m3(x * inv), round to nearest even with saturation at +-448.
 //
-// GEMM: one CTA per 128 x BN output tile (BN = 256 when D_out % 256 == 0 and that grid fills
-// two waves, else 128); both operands K-major with 128-byte swizzle (one 128-byte row = 128
-// codes = four K=32 UMMA steps), a 4-stage (BN 256) or 3-stage (BN 128) TMA ring, k-steps
-// alternating between two TMEM accumulators (two independent dependency chains), and an
-// epilogue that adds the two, applies both scales and stores bf16.  Warp 0 issues TMA, warp 1 allocates TMEM and issues UMMAs, warps 2-5 drain
-// TMEM (warp w reads lanes 32 (w % 4) .. +31).  Every wait is bounded.
+// GEMM: persistent, one CTA per SM looping over 128 x BN output tiles (BN = 256 when
+// D_out % 256 == 0 and there are at least two waves of such tiles, else 128); both operands
+// K-major with 128-byte swizzle (one 128-byte row = 128 codes = four K=32 UMMA steps), a
+// 4-stage TMA ring that runs on across tile boundaries, two accumulator sets in TMEM so that
+// the epilogue of one tile (both scales, bf16 store) overlaps the UMMAs of the next; with
+// 128-column tiles each set has two accumulation chains that the k-steps alternate between.
+// Warp 0 issues TMA, warp 1 allocates TMEM and issues UMMAs, warps 2-5 drain TMEM (warp w
+// reads lanes 32 (w % 4) .. +31).  Every wait is bounded.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -157,22 +159,29 @@ constexpr uint64_t Q_DRAIN_NS = 200ull * 1000 * 1000;
 
 template <int BN>
 struct QCfg {
-  // 256-column tiles: 4 stages, one CTA per SM; 128-column tiles: 3 stages (96 KB) so that two
-  // CTAs share an SM and one's set-up and epilogue overlap the other's UMMAs.
-  static constexpr int QST = BN == 256 ? 4 : 3;
-  static constexpr int A_BYTES = QM * QK;      // 16 KB
-  static constexpr int B_BYTES = BN * QK;      // 32 or 16 KB
+  // Persistent: one CTA per SM loops over output tiles.  Two accumulator sets in TMEM let the
+  // epilogue of one tile overlap the UMMAs of the next; with 128-column tiles each set holds
+  // two accumulation chains (k-steps alternate between them), with 256-column tiles one.
+  static constexpr int CHAINS = BN == 256 ? 1 : 2;
+  static constexpr int SET = CHAINS * BN;         // TMEM columns per accumulator set
+  static constexpr int QST = 4;
+  static constexpr int A_BYTES = QM * QK;         // 16 KB
+  static constexpr int B_BYTES = BN * QK;         // 32 or 16 KB
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int OFF_BAR = QST * STAGE;
-  static constexpr int N_BAR = 2 * QST + 2;    // full/empty per stage, accumulators done, drain
+  static constexpr int N_BAR = 2 * QST + 4 + 1;   // full/empty per stage, set full/empty x2, drain
   static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;
-  static_assert(SMEM <= 232448 && STAGE % 1024 == 0, "shared memory layout");
+  // more than half of an SM's shared memory: one CTA per SM, so the 512-column TMEM
+  // allocation never waits for another CTA
+  static_assert(SMEM > 116 * 1024 && SMEM <= 232448 && STAGE % 1024 == 0, "shared memory layout");
   static constexpr uint32_t IDESC = idesc_e4m3(QM, BN);
-  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulation chains
+  static constexpr uint32_t TMEM_COLS = 2 * SET;
+  static_assert(TMEM_COLS == 512, "two accumulator sets fill TMEM");
 };
 
 struct GemmParams {
   int32_t T, D, Dout, n_kb;
+  int32_t n_mt, n_tiles;   // row tiles; all tiles (tile t: rows (t % n_mt), columns (t / n_mt))
   const float* a_scale;
   const float* w_scale;
   __nv_bfloat16* out;
@@ -181,7 +190,7 @@ struct GemmParams {
 };
 
 template <int BN>
-__global__ void __launch_bounds__(Q_THREADS, BN == 256 ? 1 : 2)
+__global__ void __launch_bounds__(Q_THREADS, 1)
     w8a8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_w,
                      const GemmParams p) {
   using C = QCfg<BN>;
@@ -196,10 +205,9 @@ __global__ void __launch_bounds__(Q_THREADS, BN == 256 ? 1 : 2)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::N_BAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * QST, acc_bar = empty0 + 8 * QST,
-                 drain_bar = acc_bar + 8;
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * QST, accf0 = empty0 + 8 * QST,
+                 acce0 = accf0 + 16, drain_bar = acce0 + 16;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * QM, n0 = blockIdx.y * BN;
   const int n_kb = p.n_kb;
 
   if (threadIdx.x == 0) {
@@ -207,7 +215,10 @@ __global__ void __launch_bounds__(Q_THREADS, BN == 256 ? 1 : 2)
       mbar_init(full0 + 8 * i, 1);
       mbar_init(empty0 + 8 * i, 1);
     }
-    mbar_init(acc_bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(accf0 + 8 * i, 1);
+      mbar_init(acce0 + 8 * i, 128);
+    }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -223,51 +234,72 @@ __global__ void __launch_bounds__(Q_THREADS, BN == 256 ? 1 : 2)
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
 
   if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int issued = 0;
-      for (int kb = 0; kb < n_kb; ++kb) {
-        const int st = kb % QST;
-        if (!mbar_wait(empty0 + 8 * st, ((kb / QST) & 1) ^ 1, wc, 31, kb)) break;
-        mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
-        const uint32_t sa = sbase + st * C::STAGE;
-        tma_load_2d(sa, &tm_a, full0 + 8 * st, kb * QK, m0);
-        tma_load_2d(sa + C::A_BYTES, &tm_w, full0 + 8 * st, kb * QK, n0);
-        issued = kb + 1;
+      int g = 0;   // k-blocks issued over all tiles of this CTA
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < p.n_tiles; t += gridDim.x) {
+        const int m0 = (t % p.n_mt) * QM, n0 = (t / p.n_mt) * BN;
+        for (int kb = 0; kb < n_kb; ++kb, ++g) {
+          const int st = g % QST;
+          if (!mbar_wait(empty0 + 8 * st, ((g / QST) & 1) ^ 1, wc, 31, g)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
+          const uint32_t sa = sbase + st * C::STAGE;
+          tma_load_2d(sa, &tm_a, full0 + 8 * st, kb * QK, m0);
+          tma_load_2d(sa + C::A_BYTES, &tm_w, full0 + 8 * st, kb * QK, n0);
+        }
       }
-      for (int i = issued > QST ? issued - QST : 0; i < issued; ++i)
+      for (int i = g > QST ? g - QST : 0; i < g; ++i)
         mbar_wait_drain(full0 + 8 * (i % QST), (i / QST) & 1, Q_DRAIN_NS);
     }
     __syncwarp();
   } else if (warp == 1) {
+    // ------------------------------------------------------------ UMMA issuer
     if (lane == 0) {
+      int g = 0, i = 0;
       bool ok = true;
-      for (int kb = 0; kb < n_kb; ++kb) {
-        const int st = kb % QST;
-        if (!mbar_wait(full0 + 8 * st, (kb / QST) & 1, wc, 32, kb)) {
-          ok = false;
-          break;
-        }
+      for (int t = blockIdx.x; ok && t < p.n_tiles; t += gridDim.x, ++i) {
+        const int set = i & 1;
+        // the epilogue has drained this set's previous tile (tile i - 2)
+        if (!mbar_wait(acce0 + 8 * set, ((i >> 1) & 1) ^ 1, wc, 34, i)) break;
         tc_fence_after();
-        const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
-        // four K=32 steps inside the 128-byte swizzle row, alternating accumulators
+        const uint32_t acc = tmem + set * C::SET;
+        for (int kb = 0; kb < n_kb; ++kb, ++g) {
+          const int st = g % QST;
+          if (!mbar_wait(full0 + 8 * st, (g / QST) & 1, wc, 32, g)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
+          // four K=32 steps inside the 128-byte swizzle row (alternating chains for BN 128)
 #pragma unroll
-        for (int k = 0; k < QK / 32; ++k)
-          umma_f8(tmem + (k & 1) * BN, sw128_desc(sa + 32 * k, 16, 1024), sw128_desc(sb + 32 * k, 16, 1024), C::IDESC,
-                  (kb > 0 || k > 1) ? 1u : 0u);
-        tc_commit(empty0 + 8 * st);
+          for (int k = 0; k < QK / 32; ++k)
+            umma_f8(acc + (C::CHAINS == 2 ? (k & 1) * BN : 0), sw128_desc(sa + 32 * k, 16, 1024),
+                    sw128_desc(sb + 32 * k, 16, 1024), C::IDESC, (kb > 0 || k >= C::CHAINS) ? 1u : 0u);
+          tc_commit(empty0 + 8 * st);
+        }
+        if (!ok) break;
+        tc_commit(accf0 + 8 * set);
       }
-      if (ok) tc_commit(acc_bar);
       tc_commit(drain_bar);
       mbar_wait_drain(drain_bar, 0, Q_DRAIN_NS);
     }
     __syncwarp();
   } else {
+    // ------------------------------------------------------------ epilogue (warps 2-5)
     const int quarter = warp & 3;
-    const int row = m0 + quarter * 32 + lane;
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, wc, 33, 0));
-    if (ok) {
+    int i = 0;
+    for (int t = blockIdx.x; t < p.n_tiles; t += gridDim.x, ++i) {
+      const int set = i & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8 * set, (i >> 1) & 1, wc, 33, i))) break;
       tc_fence_after();
-      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      const int m0 = (t % p.n_mt) * QM, n0 = (t / p.n_mt) * BN;
+      const int row = m0 + quarter * 32 + lane;
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + set * C::SET;
       const float sa = row < p.T ? p.a_scale[row] : 0.f;
       __nv_bfloat16* orow = p.out + static_cast<size_t>(row) * p.Dout + n0;
 #pragma unroll 1
@@ -275,23 +307,29 @@ __global__ void __launch_bounds__(Q_THREADS, BN == 256 ? 1 : 2)
         uint32_t v0[32], v1[32];
         tmem_ld32(taddr + 32 * c, v0);
         tmem_wait_ld32(v0);
-        tmem_ld32(taddr + BN + 32 * c, v1);
-        tmem_wait_ld32(v1);
+        if constexpr (C::CHAINS == 2) {
+          tmem_ld32(taddr + BN + 32 * c, v1);
+          tmem_wait_ld32(v1);
+        }
         if (row < p.T) {
           const float* sw = p.w_scale + n0 + 32 * c;
           uint32_t pk[16];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const float y0 = __fmul_rn(__fmul_rn(__uint_as_float(v0[2 * i]) + __uint_as_float(v1[2 * i]), sa), sw[2 * i]);
-            const float y1 =
-                __fmul_rn(__fmul_rn(__uint_as_float(v0[2 * i + 1]) + __uint_as_float(v1[2 * i + 1]), sa), sw[2 * i + 1]);
-            pk[i] = pack_bf16x2(y0, y1);
+          for (int e = 0; e < 16; ++e) {
+            float s0 = __uint_as_float(v0[2 * e]), s1 = __uint_as_float(v0[2 * e + 1]);
+            if constexpr (C::CHAINS == 2) {
+              s0 += __uint_as_float(v1[2 * e]);
+              s1 += __uint_as_float(v1[2 * e + 1]);
+            }
+            pk[e] = pack_bf16x2(__fmul_rn(__fmul_rn(s0, sa), sw[2 * e]), __fmul_rn(__fmul_rn(s1, sa), sw[2 * e + 1]));
           }
           uint4* d4 = reinterpret_cast<uint4*>(orow + 32 * c);
 #pragma unroll
           for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
         }
       }
+      tc_fence_before();
+      mbar_arrive(acce0 + 8 * set);
     }
   }
 
@@ -324,12 +362,16 @@ cudaError_t launch_gemm_bn(const uint8_t* a_q, const float* a_scale, const uint8
   p.D = D;
   p.Dout = Dout;
   p.n_kb = D / QK;
+  p.n_mt = (T + QM - 1) / QM;
+  p.n_tiles = p.n_mt * (Dout / BN);
   p.a_scale = a_scale;
   p.w_scale = w_scale;
   p.out = out;
   p.status = status;
   p.wait_limit_ns = wait_limit_ns;
-  const dim3 grid((T + QM - 1) / QM, Dout / BN);
+  int dev_sms = 152;
+  cudaDeviceGetAttribute(&dev_sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = p.n_tiles < dev_sms ? p.n_tiles : dev_sms;
   w8a8_gemm_kernel<BN><<<grid, Q_THREADS, C::SMEM, s>>>(ta, tw, p);
   return cudaGetLastError();
 }
@@ -362,8 +404,8 @@ cudaError_t launch_w8a8_gemm(const uint8_t* a_q, const float* a_scale, const uin
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // 256-column tiles halve the activation re-reads, but a grid of under two waves of them
-  // leaves SMs idle: then take 128-column tiles (two CTAs per SM)
+  // 256-column tiles halve the activation re-reads, but with under two waves of them the
+  // last partial wave leaves SMs idle for a large share of the run: then take 128-column tiles
   const int64_t tiles256 = static_cast<int64_t>((T + QM - 1) / QM) * (Dout / 256);
   if (Dout % 256 == 0 && tiles256 >= 2 * static_cast<int64_t>(sms))
     return launch_gemm_bn<256>(a_q, a_scale, w_q, w_scale, T, D, Dout, o, status, wait_limit_ns, s);
