@@ -25,6 +25,9 @@
  *   - Kernels never spin without bound: a wait that runs out records a device
  *     error, which ispa_last_device_error() reports as ISPA_ERR_TIMEOUT.
  *   - Head dims supported: 64 and 128.  Tokens per frame P >= 1.
+ *   - Counts (queries n_q, tokens T, frames n_frames, rows) must be at least
+ *     1: an empty call is an argument error (ISPA_ERR_INVALID_ARG) and
+ *     enqueues nothing, so callers skip empty work themselves.
  *   - Threads: entry points may be called from several host threads for
  *     different rings, states and streams.  ispa_set_wait_limit_ns and the
  *     ispa_debug_* setters change process-wide settings without locking; set

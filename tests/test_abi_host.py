@@ -196,3 +196,21 @@ def test_ring_compact_validation_without_gpu():
     # frame 0 (the sink) was evicted from src (no pinned sink there): the window cannot be kept
     assert L.ispa_ring_compact(ctypes.byref(src), Window(1, 3), ctypes.byref(dst), None) == abi.ISPA_ERR_CAPACITY
     assert dst.frames_written == 0
+
+
+def test_empty_calls_are_argument_errors_without_gpu():
+    # every count must be >= 1; an empty call is rejected before anything is enqueued
+    L = abi.lib()
+    r = KVRing(2, 64, 16, 4, 0, 0, 2, 16, 16)
+    assert L.ispa_attn_full(ctypes.byref(r), 16, 16, 16, 0, 0.0, 16, None, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_attn_local(ctypes.byref(r), Window(0, 1), 16, 16, 16, 0, 0.0, 16, None,
+                             None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_attn_dual(ctypes.byref(r), Window(0, 1), 16, 16, 16, 0, 0.0, 16, 16, 16, 16, None, None,
+                            16, 1 << 20, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_kv_append(ctypes.byref(r), 16, 16, 0, None) == abi.ISPA_ERR_INVALID_ARG
+    assert r.frames_written == 2
+    st = LSState(128, 0, 0, 16)
+    assert L.ispa_ls_accumulate(ctypes.byref(st), 16, 16, 0, 16, 1 << 30, None) == abi.ISPA_ERR_INVALID_ARG
+    assert st.n_tokens == 0
+    assert L.ispa_quantize_rows_e4m3(16, 0, 128, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_linear_w8a8(16, 16, 16, 16, 0, 128, 128, 16, None) == abi.ISPA_ERR_INVALID_ARG
