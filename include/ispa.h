@@ -181,9 +181,14 @@ ISPA_API ispa_status ispa_debug_error_record(int32_t* rec8);
 ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots);
 
 /* Debug aid: per-key-tile cycle trace of the attention kernel's first CTA.
- * buf: device-accessible uint64 [n_tiles][8] (clock64 values; events 0-2 softmax
- * S-ready / max-exchanged / P-written, 3-5 UMMA warp P-seen / PV-issued /
- * next-S-issued, 6-7 TMA K / V issued).  NULL / 0 turns it off (the default). */
+ * buf: device-accessible uint64 [n_tiles][32], clock64 values of the SM, zero
+ * where an event is not recorded.  Events of key tile j:
+ *   0, 8, 9, 1, 10, 2  softmax warp 0: S_j seen, S_j loaded from TMEM, half-row
+ *                      max done, row max exchanged, exp loop done, P_j arrived;
+ *   3, 11, 4, 5        UMMA thread: P_j seen, V_j seen, PV_j issued, S_{j+2} issued;
+ *   6, 7               TMA thread: K_j issued, V_j issued;
+ *   16 + w, 24 + w     softmax warp w (0-7): P_j arrived, S_j seen.
+ * NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
 
 /* Bytes of one ring's K and V buffers together: H * cap * P * d * (2 + 2), or

@@ -149,7 +149,10 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 
 }  // namespace
 
-template <int HD, bool QK8>
+// TRACE: the instance launched while a trace buffer is set records the per-tile events of
+// ispa_debug_set_trace; the production instances contain no trace code at all (even an
+// untaken clock64 read constrains instruction scheduling: it cost 6 % here).
+template <int HD, bool QK8, bool TRACE>
 __global__ void __launch_bounds__(NTHREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kr,
                 const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_kc,
@@ -227,6 +230,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const uint32_t tmem = *tmem_slot;
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
   const int n_tiles = p.n_tiles;
+  auto tr = [&](int tile, int ev) {
+    if constexpr (TRACE) trace_event(p.trace, p.trace_tiles, tile, ev);
+  };
 
   if (warp == WARP_TMA) {
     // ------------------------------------------------------------ producer
@@ -249,7 +255,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
           tma_load_4d(sK, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0, row, 0, head);
           nk = t + 1;
-          trace_event(p.trace, p.trace_tiles, t, 6);
+          tr(t, 6);
           next_tile(p, kseg, koff);
         }
         if (t >= 1) {
@@ -262,7 +268,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
           tma_load_4d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0, row, 0, head);
           nv = j + 1;
-          trace_event(p.trace, p.trace_tiles, j, 7);
+          tr(j, 7);
           next_tile(p, vseg, voff);
         }
       }
@@ -309,8 +315,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int vs = j % C::VST;
         if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
-        trace_event(p.trace, p.trace_tiles, j, 3);
+        tr(j, 3);
         if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
+        tr(j, 11);
         tc_fence_after();
         const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
         const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
@@ -321,9 +328,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         tc_commit(b.o_done0 + 8 * (j & 1));
         tc_commit(b.v_empty0 + 8 * vs);
-        trace_event(p.trace, p.trace_tiles, j, 4);
+        tr(j, 4);
         if (j + 2 < n_tiles) ok = issue_s(j + 2);
-        trace_event(p.trace, p.trace_tiles, j, 5);
+        tr(j, 5);
       }
       // All UMMAs must have finished before TMEM is released.
       tc_commit(b.drain);
@@ -417,7 +424,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         emit(ok, p.out_loc, p.lse_loc, false, j & 1);
       }
       if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
-      if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 0);
+      if (threadIdx.x == 0) tr(j, 0);
+      if (lane == 0) tr(j, 24 + warp);
       const int valid = min(BN, p.seg[seg].count - off);
       const float sl2 = p.seg[seg].src != 0 ? sl2_chunk : sl2_ring;
       const uint64_t sl2x2 = f2_pack(sl2, sl2);
@@ -430,6 +438,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
 #pragma unroll
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
+        if (threadIdx.x == 0) tr(j, 8);
         int vloc = valid - half * HALF_COLS;   // valid columns of this half
         if (p.causal_p != 0 && p.seg[seg].src != 0) {
           // frame-causal chunk: this row sees chunk keys below the end of its own frame
@@ -448,10 +457,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           m1 = max3(m1, __uint_as_float(s[i + 2]), __uint_as_float(s[i + 3]));
         }
         mx = fmaxf(m0, m1);
+        if (threadIdx.x == 0) tr(j, 9);
       }
       x_max[(sb * 2 + half) * BM + row] = mx;
       soft_barrier();
-      if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 1);
+      if (threadIdx.x == 0) tr(j, 1);
       if (ok) {
         const float m_tile = fmaxf(mx, x_max[(sb * 2 + (half ^ 1)) * BM + row]) * sl2;
         if (j == 0) {
@@ -503,12 +513,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
           tmem_st4(pcol + 4 * c, pk);
         }
+        if (threadIdx.x == 0) tr(j, 10);
         const uint64_t acc = f2_add(acc0, acc1);
         l_run += __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(b.p_full0 + 8 * sb);
-        if (threadIdx.x == 0) trace_event(p.trace, p.trace_tiles, j, 2);
+        if (threadIdx.x == 0) tr(j, 2);
+        if (lane == 0) tr(j, 16 + warp);
       }
       next_tile(p, seg, off);
     }
@@ -530,7 +542,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
 }
 
-template <int HD, bool QK8>
+template <int HD, bool QK8, bool TRACE = false>
 static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, const CUtensorMap* tvr,
                              const CUtensorMap* tkc, const CUtensorMap* tvc, const AttnParams& p,
                              cudaStream_t s) {
@@ -539,12 +551,12 @@ static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, cons
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, QK8>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, QK8, TRACE>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_done[dev] = true;
   }
   dim3 grid((p.n_q + BM - 1) / BM, p.num_heads);
-  attn_kernel<HD, QK8><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
+  attn_kernel<HD, QK8, TRACE><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
   return cudaGetLastError();
 }
 
@@ -555,6 +567,7 @@ cudaError_t launch_attention(int head_dim, const CUtensorMap* tq, const CUtensor
     if (head_dim == 128) return launch_hd<128, true>(tq, tkr, tvr, tkc, tvc, p, s);
     return cudaErrorInvalidValue;
   }
+  if (head_dim == 128 && p.trace) return launch_hd<128, false, true>(tq, tkr, tvr, tkc, tvc, p, s);
   if (head_dim == 128) return launch_hd<128, false>(tq, tkr, tvr, tkc, tvc, p, s);
   if (head_dim == 64) return launch_hd<64, false>(tq, tkr, tvr, tkc, tvc, p, s);
   return cudaErrorInvalidValue;

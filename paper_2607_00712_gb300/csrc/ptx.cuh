@@ -112,9 +112,10 @@ __device__ __forceinline__ void heartbeat(uint32_t* hb, int idx) {
   }
 }
 
-// Debug cycle trace: tr[tile * 8 + event] = clock64() for CTA (0, 0) only.
+// Debug cycle trace: tr[tile * 32 + event] = clock64() for CTA (0, 0) only.
+constexpr int kTraceSlots = 32;
 __device__ __forceinline__ void trace_event(uint64_t* tr, int n, int tile, int ev) {
-  if (tr && tile < n && blockIdx.x == 0 && blockIdx.y == 0) tr[tile * 8 + ev] = clock64();
+  if (tr && tile < n && blockIdx.x == 0 && blockIdx.y == 0) tr[tile * kTraceSlots + ev] = clock64();
 }
 
 // Drain wait used on the abort path: ignores the abort flag, fixed limit.
