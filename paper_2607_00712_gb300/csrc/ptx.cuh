@@ -85,10 +85,10 @@ __device__ __forceinline__ void raise_abort(const WaitCtx& w, int code) {
 // Wait for the phase of `bar` with the given parity to complete.  Returns
 // false (and raises the abort flag) once the limit has passed, or as soon as
 // another role of the CTA has aborted.  `site` and `detail` identify the wait
-// in the error record.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& w, int site = 0,
-                                          int detail = 0) {
-  if (mbar_try_wait(bar, parity)) return true;
+// in the error record.  Only the first test is inlined at the call site; the
+// bounded polling loop (timer reads, abort checks, error record) is a call, so
+// the hot loops carry none of its volatile code.
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, WaitCtx w, int site, int detail) {
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -101,6 +101,11 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const W
       }
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& w, int site = 0,
+                                          int detail = 0) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, w, site, detail);
 }
 
 // Heartbeat counters in host-visible memory (debug aid): hb[0] += 1 at CTA
