@@ -187,7 +187,9 @@ ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slot
  *                      max done, row max exchanged, exp loop done, P_j arrived;
  *   3, 11, 4, 5        UMMA thread: P_j seen, V_j seen, PV_j issued, S_{j+2} issued;
  *   6, 7               TMA thread: K_j issued, V_j issued;
- *   16 + w, 24 + w     softmax warp w (0-7): P_j arrived, S_j seen.
+ *   16 + w, 24 + w     softmax warp w (0-7): P_j arrived, S_j seen;
+ *   12-15 of tile 0    once per CTA: kernel entry, TMEM allocated, Q tile landed,
+ *                      epilogue stored.
  * NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
 

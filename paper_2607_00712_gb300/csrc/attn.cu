@@ -167,6 +167,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (threadIdx.x == 0) record_error(p.status, DEVERR_LAYOUT, 0, sbase, 0, 0);
     return;
   }
+  uint64_t t_start = 0;
+  if constexpr (TRACE) t_start = clock64();
   float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [parity][half][row]
   uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
@@ -233,6 +235,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   auto tr = [&](int tile, int ev) {
     if constexpr (TRACE) trace_event(p.trace, p.trace_tiles, tile, ev);
   };
+  if constexpr (TRACE) {
+    // once per CTA, in tile 0's spare slots: 12 kernel entry, 13 TMEM allocated
+    if (threadIdx.x == 0 && p.trace && p.trace_tiles > 0 && blockIdx.x == 0 && blockIdx.y == 0) p.trace[12] = t_start;
+    if (threadIdx.x == 0) tr(0, 13);
+  }
 
   if (warp == WARP_TMA) {
     // ------------------------------------------------------------ producer
@@ -286,6 +293,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (lane == 0) {
       const uint32_t sQ = sbase + C::OFF_Q;
       bool ok = mbar_wait(b.q_full, 0, wc, 3, 0);
+      tr(0, 14);   // Q tile landed
       tc_fence_after();
       auto issue_s = [&](int j) -> bool {
         const int ks = j % C::KST;
@@ -530,6 +538,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       if (ok) tc_fence_after();
       if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false, n_tiles & 1);
       emit(ok, p.out, p.lse, p.dual != 0, n_tiles & 1);
+      if (threadIdx.x == 0) tr(0, 15);   // epilogue stored
     }
   }
 

@@ -99,6 +99,14 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
     }
     res = {k: med(f) for k, f in rows.items()}
     res["tiles traced"] = n
+    # fill and drain of the first CTA (one sample each)
+    res["CTA: entry -> TMEM allocated"] = int(t[0, 13] - t[0, 12])
+    res["CTA: TMEM allocated -> Q landed"] = int(t[0, 14] - t[0, 13])
+    res["CTA: Q landed -> S_0 seen by softmax warp 0"] = int(t[0, 0] - t[0, 14])
+    res["CTA: entry -> P_0 seen (first PV can start)"] = int(t[0, 3] - t[0, 12])
+    res["CTA: entry -> last P seen"] = int(t[n - 1, 3] - t[0, 12])
+    res["CTA: last P seen -> epilogue stored"] = int(t[0, 15] - t[n - 1, 3])
+    res["CTA: entry -> epilogue stored"] = int(t[0, 15] - t[0, 12])
     return res
 
 
