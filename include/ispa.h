@@ -152,8 +152,8 @@ ISPA_API const char* ispa_status_string(ispa_status s);
 
 /* Device error recorded by a kernel on the current device since the last
  * call (then cleared): ISPA_OK, ISPA_ERR_TIMEOUT (raw code 1), or ISPA_ERR_CUDA
- * (raw code 3: an attention CTA found its shared-memory window off a 1 KB
- * boundary and wrote nothing).  Synchronises the device with a blocking copy
+ * (raw code 3: a CTA of a tcgen05 kernel -- attention, Gram, W8A8 -- found its
+ * shared-memory window off a 1 KB boundary and wrote nothing).  Synchronises the device with a blocking copy
  * of one word.  *code (nullable, host) gets the raw code. */
 ISPA_API ispa_status ispa_last_device_error(int32_t* code);
 
@@ -180,7 +180,9 @@ ISPA_API ispa_status ispa_debug_error_record(int32_t* rec8);
  * NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots);
 
-/* Debug aid: per-key-tile cycle trace of the attention kernel's first CTA.
+/* Debug aid: per-key-tile cycle trace of CTA (0, 0) of the bf16, head_dim 128
+ * attention kernel (a separate instance of it, launched while a buffer is set;
+ * it computes the same results).
  * buf: device-accessible uint64 [n_tiles][32], clock64 values of the SM, zero
  * where an event is not recorded.  Events of key tile j:
  *   0, 8, 9, 1, 10, 2  softmax warp 0: S_j seen, S_j loaded from TMEM, half-row
