@@ -63,3 +63,14 @@ def test_reference_arm_skips_non_zero_ranks(capsys):
         warmup = 0
     bench.run_reference(A, rank=1, world=2)
     assert capsys.readouterr().out == ""
+
+
+def test_clock_rejection_rule():
+    import bench
+    ok = dict(sm_mhz=2070.0, sm_max_mhz=2070.0, reasons=[], samples=5)
+    assert not bench.clock_rejected(ok) and not bench.clock_rejected(None)
+    assert not bench.clock_rejected(dict(ok, reasons=["sw_power_cap"], sm_mhz=1900.0))
+    assert bench.clock_rejected(dict(ok, reasons=["hw_slowdown"]))
+    assert bench.clock_rejected(dict(ok, reasons=["sw_thermal_slowdown", "sw_power_cap"]))
+    assert bench.clock_rejected(dict(ok, sm_mhz=1400.0))              # stuck low, no reason
+    assert not bench.clock_rejected(dict(ok, sm_mhz=1400.0, reasons=["sw_power_cap"]))
