@@ -7,7 +7,10 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
+#include <set>
+#include <utility>
 #include <vector>
 
 #include "internal.h"
@@ -50,7 +53,7 @@ uint64_t wait_limit_ns() { return g_wait_limit; }
 namespace {
 uint32_t* g_hb = nullptr;   // host-mapped heartbeat buffer (device address), debug only
 int g_hb_slots = 0;
-int g_hb_next = 0;
+std::atomic<int> g_hb_next{0};
 }  // namespace
 
 uint64_t* g_trace = nullptr;
@@ -63,22 +66,36 @@ uint64_t* trace_buffer(int32_t* n_tiles) {
 
 uint32_t* next_heartbeat_slot(uint32_t kernel_tag) {
   if (!g_hb || g_hb_slots <= 0) return nullptr;
-  uint32_t* slot = g_hb + 4 * (g_hb_next % g_hb_slots);
-  ++g_hb_next;
+  uint32_t* slot = g_hb + 4 * (g_hb_next.fetch_add(1, std::memory_order_relaxed) % g_hb_slots);
   (void)kernel_tag;
   return slot;
 }
 
 int* device_status_ptr() {
-  static int* ptrs[64] = {};
+  static std::atomic<int*> ptrs[64] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  if (!ptrs[dev]) {
+  int* cached = ptrs[dev].load(std::memory_order_acquire);
+  if (!cached) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
-    ptrs[dev] = static_cast<int*>(p);
+    cached = static_cast<int*>(p);
+    ptrs[dev].store(cached, std::memory_order_release);
   }
-  return ptrs[dev];
+  return cached;
+}
+
+cudaError_t set_smem_limit_once(const void* func, int bytes) {
+  static std::mutex mu;
+  static std::set<std::pair<int, const void*>> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done.count({dev, func})) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done.insert({dev, func});
+  return e;
 }
 
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
@@ -400,7 +417,7 @@ ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots) {
   if ((counters == nullptr) != (n_slots <= 0)) return ISPA_ERR_INVALID_ARG;
   g_hb = counters;
   g_hb_slots = n_slots;
-  g_hb_next = 0;
+  g_hb_next.store(0, std::memory_order_relaxed);
   return ISPA_OK;
 }
 

@@ -556,13 +556,11 @@ static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, cons
                              const CUtensorMap* tkc, const CUtensorMap* tvc, const AttnParams& p,
                              cudaStream_t s) {
   using C = Cfg<HD, QK8>;
-  static bool attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, QK8, TRACE>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  {
+    const cudaError_t e = set_smem_limit_once(reinterpret_cast<const void*>(attn_kernel<HD, QK8, TRACE>), C::SMEM);
     if (e != cudaSuccess) return e;
-    attr_done[dev] = true;
   }
   dim3 grid((p.n_q + BM - 1) / BM, p.num_heads);
   attn_kernel<HD, QK8, TRACE><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);

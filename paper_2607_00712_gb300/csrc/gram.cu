@@ -617,14 +617,12 @@ __global__ void __launch_bounds__(W_THREADS, 1)
 static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
                                     float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
                                     cudaStream_t s) {
-  static bool attr_done[64] = {};
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(gram_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, W_SMEM);
+  {
+    const cudaError_t e = set_smem_limit_once(reinterpret_cast<const void*>(gram_wide_kernel), W_SMEM);
     if (e != cudaSuccess) return e;
-    attr_done[dev] = true;
   }
   // [T][D] operands viewed as (64 features, T tokens, D/64 feature blocks); one box
   // (64, GK, 4) is a 256-feature slice of GK tokens as 4 swizzled [GK][128 B] blocks
@@ -671,14 +669,12 @@ template <int BN>
 static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
                                float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
   using C = GCfg<BN>;
-  static bool attr_done[64] = {};
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(gram_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  {
+    const cudaError_t e = set_smem_limit_once(reinterpret_cast<const void*>(gram_kernel<BN>), C::SMEM);
     if (e != cudaSuccess) return e;
-    attr_done[dev] = true;
   }
   // [T][D] operands viewed as (64 features, T tokens, D/64 feature blocks): the block
   // stride (128 B) is below the token stride, so one box (64, GK, n) fetches n adjacent

@@ -53,6 +53,10 @@ struct AttnParams {
   const float* kr_scale;
 };
 
+// Raise the dynamic shared-memory limit of `func` to `bytes` on the current device, once
+// per (device, kernel); safe to call from several host threads.
+cudaError_t set_smem_limit_once(const void* func, int bytes);
+
 // Launch the attention kernel.  tensor maps are encoded by the caller.
 cudaError_t launch_attention(int head_dim, const CUtensorMap* tm_q, const CUtensorMap* tm_kr,
                              const CUtensorMap* tm_vr, const CUtensorMap* tm_kc,

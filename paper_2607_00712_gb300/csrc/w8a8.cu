@@ -346,13 +346,11 @@ cudaError_t launch_gemm_bn(const uint8_t* a_q, const float* a_scale, const uint8
                            int32_t T, int32_t D, int32_t Dout, __nv_bfloat16* out, int* status,
                            uint64_t wait_limit_ns, cudaStream_t s) {
   using C = QCfg<BN>;
-  static bool attr_done[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    const cudaError_t e = cudaFuncSetAttribute(w8a8_gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  {
+    const cudaError_t e = set_smem_limit_once(reinterpret_cast<const void*>(w8a8_gemm_kernel<BN>), C::SMEM);
     if (e != cudaSuccess) return e;
-    attr_done[dev] = true;
   }
   CUtensorMap ta, tw;
   if (!encode_tmap_2d_u8(&ta, a_q, D, T, D, QK, QM) || !encode_tmap_2d_u8(&tw, w_q, D, Dout, D, QK, BN))
