@@ -32,6 +32,28 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+
+// The tensor-map encoder below is a driver-API call.  In a host thread that has not yet made a
+// CUDA runtime call no context is current, and the encoder fails there (the runtime binds a
+// context only for its own calls).  Bind the current device's primary context first, as the
+// runtime would: a no-op when a context is already current.
+void ensure_context() {
+  static CtxGetCurrentFn get = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get = reinterpret_cast<CtxGetCurrentFn>(p);
+  });
+  CUcontext c = nullptr;
+  if (get && get(&c) == CUDA_SUCCESS && c) return;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaSetDevice(dev);
+}
+
 EncodeTiledFn encode_fn() {
   static EncodeTiledFn fn = nullptr;
   static std::once_flag once;
@@ -101,6 +123,7 @@ cudaError_t set_smem_limit_once(const void* func, int bytes) {
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                     uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                     uint32_t b2) {
+  ensure_context();
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[3] = {d0, d1, d2};
@@ -114,6 +137,7 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, 
 
 bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], const uint64_t strides3[3],
                     const uint32_t box4[4], bool u8) {
+  ensure_context();
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[4] = {dims4[0], dims4[1], dims4[2], dims4[3]};
@@ -127,6 +151,7 @@ bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], c
 
 bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
                        uint32_t b0, uint32_t b1) {
+  ensure_context();
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {d0, d1};
@@ -140,6 +165,7 @@ bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d
 
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1) {
+  ensure_context();
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {d0, d1};
