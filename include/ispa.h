@@ -28,6 +28,13 @@
  *   - Counts (queries n_q, tokens T, frames n_frames, rows) must be at least
  *     1: an empty call is an argument error (ISPA_ERR_INVALID_ARG) and
  *     enqueues nothing, so callers skip empty work themselves.
+ *   - CUDA graphs: after one eager call on a device, the attention, append, LS
+ *     accumulate, quantisation and W8A8 entry points enqueue only kernel
+ *     launches on `stream` and can be captured.  A replay reuses what the call
+ *     saw at capture time: pointers, and the ring's frames_written and hence its
+ *     key sets (an append advances frames_written on the host when it is
+ *     captured, not when it is replayed).  ispa_ls_solve and the functions that
+ *     read the device error record synchronise and cannot be captured.
  *   - Threads: entry points may be called from several host threads for
  *     different rings, states and streams.  ispa_set_wait_limit_ns and the
  *     ispa_debug_* setters change process-wide settings without locking; set
