@@ -29,8 +29,8 @@
  *     1: an empty call is an argument error (ISPA_ERR_INVALID_ARG) and
  *     enqueues nothing, so callers skip empty work themselves.
  *   - CUDA graphs: after one eager call on a device, the attention, append, LS
- *     accumulate, quantisation and W8A8 entry points enqueue only kernel
- *     launches on `stream` and can be captured.  A replay reuses what the call
+ *     accumulate / reset, quantisation and W8A8 entry points enqueue only
+ *     kernel launches and memsets on `stream` and can be captured.  A replay reuses what the call
  *     saw at capture time: pointers, and the ring's frames_written and hence its
  *     key sets (an append advances frames_written on the host when it is
  *     captured, not when it is replayed).  ispa_ls_solve and the functions that
