@@ -214,3 +214,10 @@ def test_empty_calls_are_argument_errors_without_gpu():
     assert st.n_tokens == 0
     assert L.ispa_quantize_rows_e4m3(16, 0, 128, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 0, 128, 128, 16, None) == abi.ISPA_ERR_INVALID_ARG
+
+
+def test_append_of_more_than_sixteen_frames_is_rejected_without_gpu():
+    L = abi.lib()
+    r = KVRing(2, 64, 16, 40, 0, 0, 0, 16, 16)
+    assert L.ispa_kv_append(ctypes.byref(r), 16, 16, 17, None) == abi.ISPA_ERR_CAPACITY
+    assert r.frames_written == 0

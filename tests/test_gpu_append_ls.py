@@ -167,3 +167,20 @@ def test_bounded_wait_reports_timeout():
     # the context is still usable
     x = torch.ones(4, device="cuda")
     assert float(x.sum()) == 4.0
+
+
+def test_append_sixteen_frames_the_largest_single_append():
+    H, d, P, cap = 2, 64, 24, 20
+    ring = Ring(H, d, P, cap, 1)
+    rng = np.random.default_rng(16)
+    k = synth.bf16_round(rng.standard_normal((16 * P, H, d), dtype=np.float32))
+    v = synth.bf16_round(rng.standard_normal((16 * P, H, d), dtype=np.float32))
+    ring.c.frames_written = 7                      # the 16 frames wrap around the non-sink slots
+    abi.ispa_kv_append(ring.c, bf16_tensor(k), bf16_tensor(v), 16)
+    torch.cuda.synchronize()
+    assert ring.frames_written == 23
+    kk, vv = to_f32(ring.k), to_f32(ring.v)
+    for i in range(16):
+        s = ks.ring_slot(7 + i, cap, 1)
+        assert np.array_equal(kk[:, s * P:(s + 1) * P], k[i * P:(i + 1) * P].transpose(1, 0, 2))
+        assert np.array_equal(vv[:, s * P:(s + 1) * P], v[i * P:(i + 1) * P].transpose(1, 0, 2))
