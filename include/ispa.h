@@ -190,11 +190,16 @@ ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slot
 /* Debug aid: per-key-tile cycle trace of CTA (0, 0) of the bf16, head_dim 128
  * attention kernel (a separate instance of it, launched while a buffer is set;
  * it computes the same results).
- * buf: device-accessible uint64 [n_tiles][32], clock64 values of the SM, zero
- * where an event is not recorded.  Events of key tile j:
- *   0, 8, 9, 1, 10, 2  softmax warp 0: S_j seen, S_j loaded from TMEM, half-row
- *                      max done, row max exchanged, exp loop done, P_j arrived;
+ * buf: device-accessible uint64 [n_tiles][32], clock64 values, zero where an
+ * event is not recorded.  The counters of an SM's four sub-partitions are not
+ * aligned with one another: compare stamps of warps on different sub-partitions
+ * (warp index mod 4) only through intervals each warp measures on its own.
+ * Events of key tile j:
+ *   0, 8, 9, 1, 10, 2  softmax warp 0: S_j seen, S_j loaded from TMEM, tile max
+ *                      of its half-row done, rescale decided (warp-pair barrier),
+ *                      exp loop done, P_j arrived;
  *   3, 11, 4, 5        UMMA thread: P_j seen, V_j seen, PV_j issued, S_{j+2} issued;
+ *   15 (j >= 1)        UMMA thread: K_j landed;
  *   6, 7               TMA thread: K_j issued, V_j issued;
  *   16 + w, 24 + w     softmax warp w (0-7): P_j arrived, S_j seen;
  *   12-15 of tile 0    once per CTA: kernel entry, TMEM allocated, Q tile landed,

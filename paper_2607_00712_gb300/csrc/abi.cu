@@ -253,7 +253,7 @@ ispa_status resolve(const ispa_kv_ring* r, ispa_window win, ispa_key_sets* ks) {
 // ------------------------------------------------------------ attention driver
 enum Mode { MODE_FULL, MODE_LOCAL, MODE_DUAL, MODE_HIST };
 
-int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
+int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P, int bn) {
   int tiles = 0;
   for (int i = 0; i < n; ++i) {
     AttnSeg& s = p.seg[p.n_seg++];
@@ -261,7 +261,7 @@ int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P) {
     s.start = r[i].first_slot * P;
     s.count = r[i].n_slots * P;
     s.pad = 0;
-    tiles += (s.count + kAttnBN - 1) / kAttnBN;
+    tiles += (s.count + bn - 1) / bn;
   }
   return tiles;
 }
@@ -293,6 +293,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   if (st != ISPA_OK) return st;
 
   const int H = ring->num_heads, HD = ring->head_dim, P = ring->tokens_per_frame;
+  const int bn = kAttnBN;   // keys per tile: the TMA box height of K and V and the tile count
   AttnParams p;
   memset(&p, 0, sizeof(p));
   p.n_q = n_q;
@@ -302,25 +303,25 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   int tiles = 0;
   if (mode == MODE_HIST) {
     // Eq. 10: the history set alone, no chunk
-    tiles = add_segs(p, 0, ks.hist, ks.n_hist, P);
+    tiles = add_segs(p, 0, ks.hist, ks.n_hist, P, bn);
     if (tiles == 0) return launch_empty_branch(out, lse, n_q, H, HD, stream) == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
     p.n_local_tiles = tiles;
     p.n_tiles = tiles;
   } else if (mode == MODE_FULL) {
-    tiles += add_segs(p, 0, ks.full, ks.n_full, P);
+    tiles += add_segs(p, 0, ks.full, ks.n_full, P, bn);
   } else {
-    tiles += add_segs(p, 0, ks.local, ks.n_local, P);
+    tiles += add_segs(p, 0, ks.local, ks.n_local, P, bn);
   }
   if (mode != MODE_HIST) {
     AttnSeg& s = p.seg[p.n_seg++];
     s.src = 1;
     s.start = 0;
     s.count = n_q;
-    tiles += (n_q + kAttnBN - 1) / kAttnBN;
+    tiles += (n_q + bn - 1) / bn;
   }
   if (mode != MODE_HIST) {
     p.n_local_tiles = tiles;
-    if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P);
+    if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P, bn);
     p.n_tiles = tiles;
   }
   p.dual = mode == MODE_DUAL ? 1 : 0;
@@ -352,7 +353,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const uint64_t dims_r[4] = {64, ring_tok, nb, static_cast<uint64_t>(H)};
   const uint64_t str_r[3] = {row_b, 128, row_b * ring_tok};
   const uint32_t box_q[4] = {64, static_cast<uint32_t>(kAttnBM), nb, 1};
-  const uint32_t box_k[4] = {64, static_cast<uint32_t>(kAttnBN), nb, 1};
+  const uint32_t box_k[4] = {64, static_cast<uint32_t>(bn), nb, 1};
   CUtensorMap tq, tkr, tvr, tkc, tvc;
   bool ok = encode_tmap_4d(&tvc, v_cur, dims_c, str_c, box_k) && encode_tmap_4d(&tvr, ring->v, dims_r, str_r, box_k);
   if (qk8) {

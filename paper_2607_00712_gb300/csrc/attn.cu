@@ -82,9 +82,10 @@ struct Cfg {
   static constexpr int OFF_K = Q_TILE;
   static constexpr int OFF_V = OFF_K + KST * K_TILE;
   static constexpr int OFF_X = OFF_V + VST * V_TILE;          // exchange arrays (fp32)
-  static constexpr int X_FLOATS = 2 * 2 * BM;  // max[parity][half][BM]; the epilogue reuses it
-  static constexpr int OFF_BAR = OFF_X + X_FLOATS * 4;
-  static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 6 + 1;
+  static constexpr int X_FLOATS = 2 * 2 * BM;  // [block][half][BM]: pair exchanges and the epilogue
+  static constexpr int OFF_FLAG = OFF_X + X_FLOATS * 4;  // pair status [half][quarter] (int)
+  static constexpr int OFF_BAR = OFF_FLAG + 32;
+  static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 4 + 1;
   static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;  // + tmem slot / abort flag / spare
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
@@ -96,7 +97,7 @@ struct Cfg {
 };
 
 struct Bars {
-  uint32_t q_full, k_full0, k_empty0, v_full0, v_empty0, s_full0, p_full0, o_done0, drain;
+  uint32_t q_full, k_full0, k_empty0, v_full0, v_empty0, s_full0, p_full0, drain;
 };
 
 __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& off) {
@@ -109,6 +110,23 @@ __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& of
 
 __device__ __forceinline__ void soft_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(N_SOFT) : "memory");
+}
+// Barriers of one softmax warp pair (the two warps of a TMEM lane quarter, 64 threads), ids
+// 2..5; pair_or also ORs a predicate over the pair.
+__device__ __forceinline__ void pair_sync(int id) {
+  asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory");
+}
+__device__ __forceinline__ bool pair_or(int id, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, 64, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "r"(id)
+      : "memory");
+  return r != 0;
 }
 
 // Round 32 consecutive fp32 values (times inv) to bf16 pairs.
@@ -169,7 +187,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
   uint64_t t_start = 0;
   if constexpr (TRACE) t_start = clock64();
-  float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [parity][half][row]
+  float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [block][half][row]
+  volatile int* x_flag = reinterpret_cast<volatile int*>(smem + C::OFF_FLAG);   // [half][quarter]
   uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -190,8 +209,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     b.v_empty0 = b.v_full0 + 8 * C::VST;
     b.s_full0 = b.v_empty0 + 8 * C::VST;
     b.p_full0 = b.s_full0 + 16;
-    b.o_done0 = b.p_full0 + 16;
-    b.drain = b.o_done0 + 16;
+    b.drain = b.p_full0 + 16;
   }
 
   if (threadIdx.x == 0) {
@@ -207,7 +225,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(b.s_full0 + 8 * i, 1);
       mbar_init(b.p_full0 + 8 * i, N_SOFT);
-      mbar_init(b.o_done0 + 8 * i, 1);
     }
     mbar_init(b.drain, 1);
     *abort_flag = 0;
@@ -298,6 +315,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       auto issue_s = [&](int j) -> bool {
         const int ks = j % C::KST;
         if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc, 4, j)) return false;
+        if (j > 0) tr(j, 15);   // K_j landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
         tc_fence_after();
         const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
         const uint32_t d = tmem + C::COL_S0 + (j & 1) * BN;
@@ -314,8 +332,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                     sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
           }
         }
-        tc_commit(b.s_full0 + 8 * (j & 1));
-        tc_commit(b.k_empty0 + 8 * ks);
+        tc_commit(b.s_full0 + 8 * (j & 1));   // the softmax then releases K_j's stage
         return true;
       };
       if (ok) ok = issue_s(0);
@@ -334,8 +351,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::KBOX, 1024), C::IDESC_PV,
                   (j > 0 || k > 0) ? 1u : 0u);
         }
-        tc_commit(b.o_done0 + 8 * (j & 1));
-        tc_commit(b.v_empty0 + 8 * vs);
+        tc_commit(b.v_empty0 + 8 * vs);   // V_j read, and O holds tiles 0..j
         tr(j, 4);
         if (j + 2 < n_tiles) ok = issue_s(j + 2);
         tr(j, 5);
@@ -370,13 +386,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
     // Normalise O by the full-row l and store this warp's half of the row (bf16); optional
     // LSE; optional discrepancy partial sum_d (A_full - A_loc)^2 of this head on the stored
-    // bf16 values.  Executes the same two named barriers whether or not `live`.
-    // xb = parity of the next key tile: the max-exchange block of that parity is idle (its
-    // last readers passed the previous tile's barrier) and holds the l exchange; the other
-    // block, still read by the partner warp until the first barrier below, then holds sq.
-    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc, int xb) {
-      float* x_l = x_max + (xb * 2) * BM;          // [half][row]
-      float* x_sq = x_max + ((xb ^ 1) * 2) * BM;   // [half][row]
+    // bf16 values.  Executes the same two named barriers whether or not `live`.  Block 0 of
+    // the exchange area (also used by the pair exchanges, which are complete on both sides of
+    // the pair before either warp gets here) holds l, block 1 the squared sums.
+    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc) {
+      float* x_l = x_max;             // [half][row]
+      float* x_sq = x_max + 2 * BM;   // [half][row]
       x_l[half * BM + row] = l_run;
       soft_barrier();
       const float l_row = l_run + x_l[(half ^ 1) * BM + row];
@@ -423,107 +438,146 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
     };
 
+    const int pair_id = 2 + quarter;   // named barrier of the warp pair (quarter, quarter + 4)
+    // O holds tiles 0..j once PV_j has completed: the commit that frees V_j's stage.
+    auto wait_o = [&](int j, int site) {
+      return warp_ok(mbar_wait(b.v_empty0 + 8 * (j % C::VST), (j / C::VST) & 1, wc, site, j));
+    };
+    // Exchange a value and the status within the warp pair; returns the partner's value and
+    // whether both warps are ok.  Two pair barriers: the slots are free again on return.
+    auto pair_exchange = [&](float v, float& other) {
+      x_max[half * BM + row] = v;
+      if (lane == 0) x_flag[half * 4 + quarter] = ok ? 1 : 0;
+      pair_sync(pair_id);
+      other = x_max[(half ^ 1) * BM + row];
+      const bool both = ok && x_flag[(half ^ 1) * 4 + quarter] != 0;
+      pair_sync(pair_id);
+      return both;
+    };
+    // P = exp2(s * sl2 - m) for this thread's HALF_COLS scores, stored packed (bf16 pairs) at
+    // pcol as it is computed; returns the row-sum share.
+    auto exps_store = [&](const uint32_t* s, float sl2, float m, uint32_t pcol) {
+      const float mm = m == -INFINITY ? 0.f : m;   // no visible key yet: every P is 0
+      const uint64_t negm = f2_pack(-mm, -mm);
+      const uint64_t sl2x2 = f2_pack(sl2, sl2);
+      uint64_t acc0 = 0, acc1 = 0;
+#pragma unroll
+      for (int c = 0; c < P_HALF / 4; ++c) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int e = 8 * c + 2 * k;
+          const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), sl2x2, negm);
+          const float e0 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x)));
+          const float e1 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x >> 32)));
+          if (k & 1) acc1 = f2_add(acc1, f2_pack(e0, e1));
+          else acc0 = f2_add(acc0, f2_pack(e0, e1));
+          pk[k] = pack_bf16x2(e0, e1);
+        }
+        tmem_st4(pcol + 4 * c, pk);
+      }
+      const uint64_t acc = f2_add(acc0, acc1);
+      return __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
+    };
+    // maximum of this thread's scores: eight independent chains (the max is on the critical path)
+    auto raw_max = [&](const uint32_t* s) {
+      float m[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) m[k] = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < HALF_COLS; i += 2) {
+        const int k = (i / 2) & 7;
+        m[k] = max3(m[k], __uint_as_float(s[i]), __uint_as_float(s[i + 1]));
+      }
+      return fmaxf(fmaxf(fmaxf(m[0], m[1]), fmaxf(m[2], m[3])), fmaxf(fmaxf(m[4], m[5]), fmaxf(m[6], m[7])));
+    };
+
+    // Every warp walks every tile and executes the same barriers whether or not it is ok:
+    // the pair barriers of each tile, the snapshot and the epilogue.
     for (int j = 0; j < n_tiles; ++j) {
       const int sb = j & 1;
       if (p.dual && j == p.n_local_tiles && j > 0) {
         // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
-        if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 7, j));
+        if (ok) ok = wait_o(j - 1, 7);
         if (ok) tc_fence_after();
-        emit(ok, p.out_loc, p.lse_loc, false, j & 1);
+        emit(ok, p.out_loc, p.lse_loc, false);
       }
       if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
+      if (ok && warp == 0 && lane == 0) mbar_arrive(b.k_empty0 + 8 * (j % C::KST));   // S_j done: K_j read
       if (threadIdx.x == 0) tr(j, 0);
       if (lane == 0) tr(j, 24 + warp);
-      const int valid = min(BN, p.seg[seg].count - off);
+      int vloc = min(BN, p.seg[seg].count - off) - half * HALF_COLS;   // valid columns of this half
+      if (p.causal_p != 0 && p.seg[seg].src != 0) {
+        // frame-causal chunk: this row sees chunk keys below the end of its own frame
+        const int kc0 = p.seg[seg].start + off + half * HALF_COLS;   // chunk index of column 0
+        vloc = min(vloc, (qrow / p.causal_p + 1) * p.causal_p - kc0);
+      }
       const float sl2 = p.seg[seg].src != 0 ? sl2_chunk : sl2_ring;
-      const uint64_t sl2x2 = f2_pack(sl2, sl2);
-      uint32_t s[HALF_COLS];
-      float mx = -INFINITY;
-      if (ok) {
+      const uint32_t scol = trow + C::COL_S0 + sb * BN + half * HALF_COLS;
+      // load this half's scores (masked columns -inf)
+      auto load_s = [&](uint32_t* s) {
         tc_fence_after();
-        const uint32_t scol = trow + C::COL_S0 + sb * BN + half * HALF_COLS;
 #pragma unroll
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
 #pragma unroll
         for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
-        if (threadIdx.x == 0) tr(j, 8);
-        int vloc = valid - half * HALF_COLS;   // valid columns of this half
-        if (p.causal_p != 0 && p.seg[seg].src != 0) {
-          // frame-causal chunk: this row sees chunk keys below the end of its own frame
-          const int kc0 = p.seg[seg].start + off + half * HALF_COLS;   // chunk index of column 0
-          vloc = min(vloc, (qrow / p.causal_p + 1) * p.causal_p - kc0);
-        }
         if (vloc < HALF_COLS) {
 #pragma unroll
           for (int i = 0; i < HALF_COLS; ++i)
             if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
         }
-        float m0 = -INFINITY, m1 = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < HALF_COLS; i += 4) {
-          m0 = max3(m0, __uint_as_float(s[i + 0]), __uint_as_float(s[i + 1]));
-          m1 = max3(m1, __uint_as_float(s[i + 2]), __uint_as_float(s[i + 3]));
-        }
-        mx = fmaxf(m0, m1);
-        if (threadIdx.x == 0) tr(j, 9);
-      }
-      x_max[(sb * 2 + half) * BM + row] = mx;
-      soft_barrier();
-      if (threadIdx.x == 0) tr(j, 1);
+      };
+      // P_j overwrites the first 88 columns of S_j (this half's 44 packed columns), so both
+      // halves of the pair must have read their scores first: the pair barrier below orders it.
+      const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
+      uint32_t s[HALF_COLS];
+      float mx = -INFINITY;
       if (ok) {
-        const float m_tile = fmaxf(mx, x_max[(sb * 2 + (half ^ 1)) * BM + row]) * sl2;
-        if (j == 0) {
-          m_run = m_tile;
-        } else if (__any_sync(0xffffffffu, m_tile > m_run + RESCALE_THRESHOLD)) {
-          // Lazy rescale, decided per warp (the TMEM accesses are warp-collective; the
-          // partner warp of the same rows takes the same decision): O holds PV of tiles
-          // 0..j-1 once PV_{j-1} has completed.  Lanes whose max did not grow keep alpha = 1.
-          ok = warp_ok(mbar_wait(b.o_done0 + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wc, 9, j));
+        load_s(s);
+        if (threadIdx.x == 0) tr(j, 8);
+        mx = raw_max(s);
+      }
+      if (threadIdx.x == 0) tr(j, 9);
+      if (j == 0) {
+        // first tile: the row max comes from both halves
+        float mo;
+        ok = pair_exchange(mx, mo);
+        m_run = fmaxf(mx, mo) * sl2;
+      } else {
+        // the running max stands unless the tile's max exceeds it by more than 2^8 somewhere in
+        // the pair's rows (rare); then O is rescaled first
+        const bool need = ok && mx * sl2 > m_run + RESCALE_THRESHOLD;
+        if (pair_or(pair_id, need || !ok)) {
+          float mo;
+          ok = pair_exchange(mx, mo);
+          // O holds PV of tiles 0..j-1 once PV_j-1 has completed; lanes whose max did not grow
+          // keep alpha = 1.
+          if (ok) ok = wait_o(j - 1, 9);
           if (ok) {
             tc_fence_after();
-            const float m_new = fmaxf(m_run, m_tile);
-            const float alpha = ex2_approx(m_run - m_new);
+            const float m_new = fmaxf(m_run, fmaxf(mx, mo) * sl2);
+            const float alpha = m_new == m_run ? 1.f : ex2_approx(m_run - m_new);
             l_run *= alpha;
 #pragma unroll 1
-            for (int c = 0; c < C::O_HALF / 32; ++c) {
-              uint32_t r[32];
-              const uint32_t ocol = trow + C::COL_O + half * C::O_HALF + 32 * c;
-              tmem_ld32(ocol, r);
-              tmem_wait_ld32(r);
+            for (int c = 0; c < C::O_HALF / 8; ++c) {
+              uint32_t r[8];
+              const uint32_t ocol = trow + C::COL_O + half * C::O_HALF + 8 * c;
+              tmem_ld8(ocol, r);
+              tmem_wait_ld8(r);
 #pragma unroll
-              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-              tmem_st32(ocol, r);
+              for (int i = 0; i < 8; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+              tmem_st4(ocol, r);
+              tmem_st4(ocol + 4, r + 4);
             }
             tmem_wait_st();
             m_run = m_new;
           }
         }
       }
-      // P_j overwrites S_j in buffer sb: both halves have copied their S columns out
-      // (the max exchange above is a barrier), and PV_{j-2}, the last reader of this
-      // buffer's previous P, precedes S_j in the UMMA stream.
+      if (threadIdx.x == 0) tr(j, 1);
       if (ok) {
-        const uint64_t negm = f2_pack(-m_run, -m_run);
-        uint64_t acc0 = 0, acc1 = 0;
-        const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
-#pragma unroll
-        for (int c = 0; c < P_HALF / 4; ++c) {
-          uint32_t pk[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int e = 8 * c + 2 * k;
-            const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[e]), __uint_as_float(s[e + 1])), sl2x2, negm);
-            const float e0 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x)));
-            const float e1 = ex2_approx(__uint_as_float(static_cast<uint32_t>(x >> 32)));
-            if (k & 1) acc1 = f2_add(acc1, f2_pack(e0, e1));
-            else acc0 = f2_add(acc0, f2_pack(e0, e1));
-            pk[k] = pack_bf16x2(e0, e1);
-          }
-          tmem_st4(pcol + 4 * c, pk);
-        }
+        l_run += exps_store(s, sl2, m_run, pcol);
         if (threadIdx.x == 0) tr(j, 10);
-        const uint64_t acc = f2_add(acc0, acc1);
-        l_run += __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(b.p_full0 + 8 * sb);
@@ -533,11 +587,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       next_tile(p, seg, off);
     }
     {
-      const int jl = n_tiles - 1;
-      if (ok) ok = warp_ok(mbar_wait(b.o_done0 + 8 * (jl & 1), (jl >> 1) & 1, wc, 11, jl));
+      if (ok) ok = wait_o(n_tiles - 1, 11);
       if (ok) tc_fence_after();
-      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false, n_tiles & 1);
-      emit(ok, p.out, p.lse, p.dual != 0, n_tiles & 1);
+      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
+      emit(ok, p.out, p.lse, p.dual != 0);
       if (threadIdx.x == 0) tr(0, 15);   // epilogue stored
     }
   }

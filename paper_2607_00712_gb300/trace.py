@@ -75,7 +75,7 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
         abi.ispa_debug_set_trace(None, 0)
     t = buf.view(n_tiles, SLOTS).cpu().numpy().astype("int64")
     n = int((t[:, 3] != 0).sum())
-    J = list(range(10, n - 10)) if n > 30 else list(range(2, max(n - 2, 3)))
+    J = list(range(10, n - 10)) if n > 30 else list(range(3, max(n - 4, 4)))
 
     def med(f):
         return int(statistics.median(f(j) for j in J))
@@ -83,19 +83,22 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
     last_arrive = lambda j: max(t[j, 16 + w] for w in range(8))  # noqa: E731
     rows = {
         "period (UMMA thread sees P_j -> sees P_j+1)": lambda j: t[j + 1, 3] - t[j, 3],
-        "UMMA: S_j+2 issued -> sees P_j+1": lambda j: t[j + 1, 3] - t[j, 5],
         "UMMA: sees P_j -> sees V_j": lambda j: t[j, 11] - t[j, 3],
-        "UMMA: sees V_j -> PV_j issued (11 UMMAs, issue blocks)": lambda j: t[j, 4] - t[j, 11],
-        "UMMA: PV_j issued -> S_j+2 issued (8 UMMAs)": lambda j: t[j, 5] - t[j, 4],
+        "UMMA: sees V_j -> PV_j issued (11 UMMAs)": lambda j: t[j, 4] - t[j, 11],
+        "UMMA: PV_j issued -> K_j+2 landed": lambda j: t[j + 2, 15] - t[j, 4],
+        "UMMA: K_j+2 landed -> S_j+2 issued (8 UMMAs)": lambda j: t[j, 5] - t[j + 2, 15],
+        "UMMA: S_j+2 issued -> sees P_j+1": lambda j: t[j + 1, 3] - t[j, 5],
+        "S_j+2 issued -> softmax warp 0 sees it (clocks of two sub-partitions)": lambda j: t[j + 2, 0] - t[j, 5],
         "softmax w0: S_j seen -> loaded": lambda j: t[j, 8] - t[j, 0],
-        "softmax w0: loaded -> half-row max": lambda j: t[j, 9] - t[j, 8],
-        "softmax w0: half-row max -> row max exchanged": lambda j: t[j, 1] - t[j, 9],
-        "softmax w0: exchanged -> exp loop done": lambda j: t[j, 10] - t[j, 1],
+        "softmax w0: loaded -> tile max": lambda j: t[j, 9] - t[j, 8],
+        "softmax w0: tile max -> rescale decided (pair barrier)": lambda j: t[j, 1] - t[j, 9],
+        "softmax w0: rescale decided -> exp loop done": lambda j: t[j, 10] - t[j, 1],
         "softmax w0: exp loop done -> P_j arrived": lambda j: t[j, 2] - t[j, 10],
         "softmax w0: S_j seen -> P_j arrived": lambda j: t[j, 2] - t[j, 0],
+        "softmax w0: P_j arrived -> S_j+1 seen (waiting for S)": lambda j: t[j + 1, 0] - t[j, 2],
         "spread of S_j seen over the 8 softmax warps": lambda j: max(t[j, 24 + w] for w in range(8)) - min(
             t[j, 24 + w] for w in range(8)),
-        "last softmax warp's P_j arrival -> UMMA sees P_j": lambda j: t[j, 3] - last_arrive(j),
+        "last softmax warp's P_j arrival -> UMMA sees P_j (two clocks)": lambda j: t[j, 3] - last_arrive(j),
     }
     res = {k: med(f) for k, f in rows.items()}
     res["tiles traced"] = n

@@ -49,15 +49,21 @@ def test_trace_instance_matches_production_and_orders_events(mode):
     assert n >= 2 and np.all(t[:n, 3] != 0) and np.all(t[n:, :] == 0)
     for j in range(n):
         e = t[j]
-        # softmax warp 0: S seen <= loaded <= half-row max <= exchanged <= exp done <= P arrived
+        # softmax warp 0: S seen <= loaded <= P computed <= rescale decided <= P stored <= arrived
         assert e[0] <= e[8] <= e[9] <= e[1] <= e[10] <= e[2], (j, e[:12])
-        # UMMA thread: P seen <= V seen <= PV issued <= next S issued (when there is one)
-        assert e[3] <= e[11] <= e[4], (j, e[:12])
-        if j + 2 < n:
-            assert e[4] <= e[5], (j, e[:12])
+        # UMMA thread: P seen <= V seen <= PV issued <= the next S issued
+        assert e[3] <= e[11] <= e[4] <= e[5], (j, e[:12])
         # TMA thread issued K_j before the UMMA thread saw P_j, V_j before PV_j was issued
         assert e[6] <= e[3] and e[7] <= e[4], (j, e[:12])
         # every softmax warp saw S_j and published P_j (each stamp follows its own arrive, so it
         # is not ordered against the UMMA thread's view of the barrier)
         assert np.all(e[24:32] != 0) and np.all(e[16:24] != 0)
         assert np.all(e[16:24] >= e[24:32])
+        if j >= 1:
+            # slot 15 (tiles >= 1): the UMMA thread saw K_j land after the TMA thread issued it;
+            # S_1 goes out before the first PV, S_j (j >= 2) right after PV_j-2
+            assert e[6] <= e[15], (j, e[15])
+            if j >= 2:
+                assert t[j - 2, 4] <= e[15] <= t[j - 2, 5], (j, e[15])
+            else:
+                assert e[15] <= t[0, 3], (j, e[15])
