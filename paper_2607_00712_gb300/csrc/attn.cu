@@ -85,7 +85,7 @@ struct Cfg {
   static constexpr int X_FLOATS = 2 * 2 * BM;  // [block][half][BM]: pair exchanges and the epilogue
   static constexpr int OFF_FLAG = OFF_X + X_FLOATS * 4;  // pair status [half][quarter] (int)
   static constexpr int OFF_BAR = OFF_FLAG + 32;
-  static constexpr int N_BAR = 1 + 2 * KST + 2 * VST + 4 + 1;
+  static constexpr int N_BAR = 1 + KST + 2 * VST + 4 + 1;
   static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;  // + tmem slot / abort flag / spare
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
@@ -97,7 +97,7 @@ struct Cfg {
 };
 
 struct Bars {
-  uint32_t q_full, k_full0, k_empty0, v_full0, v_empty0, s_full0, p_full0, drain;
+  uint32_t q_full, k_full0, v_full0, v_empty0, s_full0, p_full0, drain;
 };
 
 __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& off) {
@@ -204,8 +204,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const uint32_t b0 = smem_u32(bar_mem);
     b.q_full = b0;
     b.k_full0 = b0 + 8 * 1;
-    b.k_empty0 = b.k_full0 + 8 * C::KST;
-    b.v_full0 = b.k_empty0 + 8 * C::KST;
+    b.v_full0 = b.k_full0 + 8 * C::KST;
     b.v_empty0 = b.v_full0 + 8 * C::VST;
     b.s_full0 = b.v_empty0 + 8 * C::VST;
     b.p_full0 = b.s_full0 + 16;
@@ -216,7 +215,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     mbar_init(b.q_full, 1);
     for (int i = 0; i < C::KST; ++i) {
       mbar_init(b.k_full0 + 8 * i, 1);
-      mbar_init(b.k_empty0 + 8 * i, 1);
     }
     for (int i = 0; i < C::VST; ++i) {
       mbar_init(b.v_full0 + 8 * i, 1);
@@ -265,8 +263,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
       tma_load_4d(sQ, &tm_q, b.q_full, 0, q0, 0, head);
       // Loads are issued in the order their stages free up: the UMMA stream is
-      // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so stages free as K_t (after S_{t-KST}) then
-      // V_{t-1} (after PV_{t-1-VST}); V therefore trails K by one tile.
+      // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so K_t goes out once S_t-2 has completed and
+      // V_{t-1} once PV_{t-1-VST} has; V therefore trails K by one tile.
       int kseg = 0, koff = 0, vseg = 0, voff = 0;
       int nk = 0, nv = 0;  // K and V tiles issued
       for (int t = 0; t <= n_tiles; ++t) {
@@ -274,7 +272,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           const bool chunk = p.seg[kseg].src != 0;
           const int row = p.seg[kseg].start + koff;
           const int ks = t % C::KST;
-          if (!mbar_wait(b.k_empty0 + 8 * ks, ((t / C::KST) & 1) ^ 1, wc, 1, t)) break;
+          // K_t's stage held K_t-KST; S_t-2 complete means K_t-2 (and every older K) has been
+          // read.  S_t cannot complete before K_t lands, so this barrier is never a phase ahead.
+          if (t >= 2 && !mbar_wait(b.s_full0 + 8 * ((t - 2) & 1), ((t - 2) >> 1) & 1, wc, 1, t)) break;
           mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::K_TILE);
           const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
           tma_load_4d(sK, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0, row, 0, head);
@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                     sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
           }
         }
-        tc_commit(b.s_full0 + 8 * (j & 1));   // the softmax then releases K_j's stage
+        tc_commit(b.s_full0 + 8 * (j & 1));   // also tells the TMA thread that K_j has been read
         return true;
       };
       if (ok) ok = issue_s(0);
@@ -503,7 +503,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         emit(ok, p.out_loc, p.lse_loc, false);
       }
       if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
-      if (ok && warp == 0 && lane == 0) mbar_arrive(b.k_empty0 + 8 * (j % C::KST));   // S_j done: K_j read
       if (threadIdx.x == 0) tr(j, 0);
       if (lane == 0) tr(j, 24 + warp);
       int vloc = min(BN, p.seg[seg].count - off) - half * HALF_COLS;   // valid columns of this half
