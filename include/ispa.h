@@ -207,6 +207,13 @@ ISPA_API ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slot
  * NULL / 0 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
 
+/* Debug aid for the timeout path: while tile >= 0, the TMA thread of every attention CTA
+ * stops before loading key tile `tile` (it issues nothing more and drains what it issued),
+ * so the UMMA thread's wait for that tile runs out after the wait limit and the CTA leaves
+ * through its abort path, recording ISPA_ERR_TIMEOUT.  CTAs with fewer tiles run normally.
+ * Nothing faults: the missing load simply never arrives.  -1 turns it off (the default). */
+ISPA_API ispa_status ispa_debug_drop_k_tile(int32_t tile);
+
 /* Bytes of one ring's K and V buffers together: H * cap * P * d * (2 + 2), or
  * * (1 + 2) with e4m3 keys. */
 ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);

@@ -76,6 +76,7 @@ _SIGS = {
     "ispa_debug_error_record": (c_int32, [POINTER(c_int32)]),
     "ispa_debug_set_heartbeat": (c_int32, [c_void_p, c_int32]),
     "ispa_debug_set_trace": (c_int32, [c_void_p, c_int32]),
+    "ispa_debug_drop_k_tile": (c_int32, [c_int32]),
     "ispa_ring_bytes": (c_size_t, [POINTER(KVRing)]),
     "ispa_ring_slot": (c_int32, [POINTER(KVRing), c_int64]),
     "ispa_window_resolve": (c_int32, [POINTER(KVRing), Window, POINTER(KeySets)]),
@@ -200,6 +201,10 @@ def ispa_debug_set_heartbeat(counters, n_slots: int) -> None:
 
 def ispa_debug_set_trace(buf, n_tiles: int) -> None:
     _check(lib().ispa_debug_set_trace(_ptr(buf), n_tiles), "ispa_debug_set_trace")
+
+
+def ispa_debug_drop_k_tile(tile: int) -> None:
+    _check(lib().ispa_debug_drop_k_tile(tile), "ispa_debug_drop_k_tile")
 
 
 def ispa_ring_bytes(ring: KVRing) -> int:

@@ -80,6 +80,7 @@ std::atomic<int> g_hb_next{0};
 
 uint64_t* g_trace = nullptr;
 int32_t g_trace_tiles = 0;
+int32_t g_drop_k_tile = -1;
 
 uint64_t* trace_buffer(int32_t* n_tiles) {
   *n_tiles = g_trace_tiles;
@@ -338,6 +339,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   if (!p.status) return ISPA_ERR_CUDA;
   p.heartbeat = next_heartbeat_slot(1);
   p.trace = trace_buffer(&p.trace_tiles);
+  p.drop_k_tile = g_drop_k_tile;
 
   // Every map views a [rows][d] bf16 operand as (64 columns, rows, d/64 column blocks, heads):
   // the column-block stride (128 B) is smaller than the row stride, so one box of
@@ -437,6 +439,12 @@ ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles) {
   if ((buf == nullptr) != (n_tiles <= 0)) return ISPA_ERR_INVALID_ARG;
   g_trace = buf;
   g_trace_tiles = n_tiles;
+  return ISPA_OK;
+}
+
+ispa_status ispa_debug_drop_k_tile(int32_t tile) {
+  if (tile < -1) return ISPA_ERR_INVALID_ARG;
+  g_drop_k_tile = tile;
   return ISPA_OK;
 }
 

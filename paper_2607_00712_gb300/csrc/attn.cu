@@ -268,6 +268,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int kseg = 0, koff = 0, vseg = 0, voff = 0;
       int nk = 0, nv = 0;  // K and V tiles issued
       for (int t = 0; t <= n_tiles; ++t) {
+        if (t == p.drop_k_tile) break;   // debug: this load never goes out (timeout-path test)
         if (t < n_tiles) {
           const bool chunk = p.seg[kseg].src != 0;
           const int row = p.seg[kseg].start + koff;

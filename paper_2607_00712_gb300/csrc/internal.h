@@ -46,7 +46,7 @@ struct AttnParams {
   uint32_t* heartbeat;     // debug counters (host-mapped) or null
   uint64_t* trace;         // debug per-tile cycle trace of CTA (0,0) or null: [tile][8]
   int32_t trace_tiles;
-  int32_t pad2;
+  int32_t drop_k_tile;     // debug: key tile the TMA thread never loads (-1: none)
   // 8-bit Q K^T (null for bf16 Q and K): per-head e4m3 code scales of q, chunk keys, ring keys
   const float* q_scale;
   const float* kc_scale;
