@@ -17,29 +17,35 @@
 // one box (64, tile rows, d/64, 1) with 128-byte swizzle fetches a whole Q, K or V
 // tile in one request as d/64 consecutive [rows][128 B] blocks, which is the
 // K-major (Q, K) and MN-major (V) UMMA operand layout.
-// CTA = one head x one tile of 128 queries, key tiles of 176 keys; 320 threads:
+// CTA = one head x one tile of 128 queries, key tiles of 192 keys; 320 threads:
 //   warps 0-7  softmax: warp w owns query rows 32(w%4)..+31 (its TMEM lane
-//              quarter) and the score columns 88(w/4)..+87 of every key tile,
-//              so each row's 176 scores are split over two warps that swap
-//              their partial row maxima through shared memory once per tile;
+//              quarter) and the score columns 96(w/4)..+95 of every key tile,
+//              so each row's 192 scores are split over a warp pair (w, w+4) on
+//              one SM sub-partition;
 //   warp 8     TMA producer (Q once, then K/V tiles into staged rings);
 //   warp 9     TMEM allocator and UMMA issuer.
-// TMEM columns: S0 [0,176) S1 [176,352) O [352,352+d).
-// Shared memory (d = 128): Q 32 KB, two K and two V stages of 44 KB, 2 KB of
-// row-max exchange (reused by the epilogue), barriers: 215,184 bytes.
-// Per key tile j: S_j = Q K_j^T (SS-UMMA, M=128 N=176, fp32 in TMEM) -> softmax
-// warps read S_j, update the row max (lazy rescale of O only when the max grows
-// by more than 2^8), write P_j = exp2(.) as bf16 over the first 88 columns of
-// S_j's own buffer -> O += P_j V_j (TS-UMMA: A operand read from TMEM).  S is
-// double buffered so S_{j+1} runs on the tensor cores while the softmax warps
-// work on S_j; S_{j+2} overwrites P_j only after PV_j, which the in-order
-// execution of one thread's UMMAs guarantees.  176-key tiles put more work in
-// each UMMA instruction than 128 (the per-instruction cost, not the work, bounds
-// 128x128x16 UMMAs here).  192-key tiles (S0 + S1 + O = all 512 columns) measured
-// about 1% slower: the PV chain (11 vs 12 dependent N=128 UMMAs) sets the pace.
+// TMEM columns: S0 [0,192) S1 [192,384) O [384,384+d).
+// Shared memory (d = 128): Q 32 KB, two K and two V stages of 48 KB, 2 KB of
+// exchange arrays, the pair status words and barriers: 231,568 bytes.
+// Per key tile j: S_j = Q K_j^T (SS-UMMA, M=128 N=192, fp32 in TMEM), one commit
+// (S_j done, which also tells the TMA thread that K_j has been read) -> the softmax
+// warps read S_j, take the tile max of their half-row, and meet their partner at one
+// 64-thread reducing barrier (bar.red.or) that orders both halves' score reads
+// before either half's P stores and carries the rescale decision (lazy: O is
+// rescaled only when the max grows by more than 2^8, rarely) and the pair's abort
+// status; they write P_j = exp2(.) as bf16 over the first 96 columns of S_j's own
+// buffer -> O += P_j V_j (TS-UMMA: A operand read from TMEM), one commit (V_j's
+// stage free, O holds tiles 0..j).  S is double buffered so S_{j+1} runs on the
+// tensor cores while the softmax warps work on S_j; S_{j+2} overwrites P_j only
+// after PV_j, which the in-order execution of one thread's UMMAs guarantees.
+// The tensor pipe runs a continuous UMMA stream at full rate; what a tile costs
+// beyond that is per-tile latency (barrier hand-offs, the TMA latency of K, the
+// softmax warps' TMEM loads), which long tiles amortise: 192-key tiles measured
+// ahead of 176 (F-layer even, L-layer and dual 0.7-0.8 %, 8-bit Q K^T 4 %), and
+// every 128-key structure tried measured 15-22 % slower.
 //
-// Every wait is bounded; after a timeout the softmax warps keep executing
-// their named barriers (without touching TMEM) so no warp is left behind.
+// Every wait is bounded; after a timeout the softmax warps skip their TMEM work but
+// keep walking the tiles through the same barriers, so no warp is left behind.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -72,7 +78,7 @@ struct Cfg {
   static_assert(!QK8 || HD == 128, "8-bit Q K^T is built for head_dim 128");
   static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per bf16 tile row
   static constexpr int QBOX = BM * 128;         // [128 rows][64 bf16] = 16 KB
-  static constexpr int KBOX = BN * 128;         // [176 rows][64 bf16] = 22 KB
+  static constexpr int KBOX = BN * 128;         // [192 rows][64 bf16] = 24 KB
   static constexpr int Q_TILE = QK8 ? BM * HD : NBOX * QBOX;
   static constexpr int K_TILE = QK8 ? BN * HD : NBOX * KBOX;
   static constexpr int V_TILE = NBOX * KBOX;
@@ -527,7 +533,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
         }
       };
-      // P_j overwrites the first 88 columns of S_j (this half's 44 packed columns), so both
+      // P_j overwrites the first 96 columns of S_j (this half's 48 packed columns), so both
       // halves of the pair must have read their scores first: the pair barrier below orders it.
       const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
       uint32_t s[HALF_COLS];

@@ -23,7 +23,7 @@ struct AttnSeg {
 
 constexpr int kMaxSegs = 8;
 constexpr int kAttnBM = 128;  // queries per attention CTA
-constexpr int kAttnBN = 176;  // keys per attention tile (TMA box rows of the K/V maps)
+constexpr int kAttnBN = 192;  // keys per attention tile (TMA box rows of the K/V maps)
 
 struct AttnParams {
   int32_t n_q;

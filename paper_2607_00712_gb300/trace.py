@@ -84,7 +84,7 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
     rows = {
         "period (UMMA thread sees P_j -> sees P_j+1)": lambda j: t[j + 1, 3] - t[j, 3],
         "UMMA: sees P_j -> sees V_j": lambda j: t[j, 11] - t[j, 3],
-        "UMMA: sees V_j -> PV_j issued (11 UMMAs)": lambda j: t[j, 4] - t[j, 11],
+        "UMMA: sees V_j -> PV_j issued (12 UMMAs)": lambda j: t[j, 4] - t[j, 11],
         "UMMA: PV_j issued -> K_j+2 landed": lambda j: t[j + 2, 15] - t[j, 4],
         "UMMA: K_j+2 landed -> S_j+2 issued (8 UMMAs)": lambda j: t[j, 5] - t[j + 2, 15],
         "UMMA: S_j+2 issued -> sees P_j+1": lambda j: t[j + 1, 3] - t[j, 5],

@@ -48,7 +48,7 @@ def _run(st, mode):
 
 @pytest.mark.parametrize("mode,drop", [("full", 3), ("dual", 3), ("dual", 7)])
 def test_attention_timeout_is_reported_and_recoverable(mode, drop):
-    # 7 past frames of 200 tokens + a 2-frame chunk: 1800 keys in 11 key tiles of 176; the dual
+    # 7 past frames of 200 tokens + a 2-frame chunk: 1800 keys in 11 key tiles of 192; the dual
     # pass's local set (2 frames + the chunk: 3 + 3 tiles) comes first, so a drop at tile 3
     # falls before its A_loc snapshot and one at tile 7 after it
     st = Step(8080, P=200, H=3, d=128, n_past=7, n_chunk_frames=2, capacity=8)
