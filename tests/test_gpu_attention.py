@@ -170,15 +170,19 @@ def test_config1_sampled_rows():
     assert np.isfinite(g["disc"]).all()
 
 
-@pytest.mark.parametrize("boost", [3.0, 6.0])
-def test_running_max_rescale_path(boost):
-    # A late frame whose keys are scaled up makes the running row max jump by more than
-    # 2^8 for some rows (boost 3: some lanes of a warp, boost 6: nearly all), exercising the
-    # lazy O rescale in TMEM, including warps where only part of the lanes need it.
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("boost,frames", [(3.0, (4, 5)), (6.0, (4, 5)), (6.0, (5,))])
+def test_running_max_rescale_path(boost, frames, d):
+    # Late frames whose keys are scaled up make the running row max jump by more than 2^8 for
+    # some rows (boost 3: some lanes of a warp, boost 6: nearly all), exercising the lazy O
+    # rescale in TMEM, including warps where only part of the lanes need it.  The 6 past frames
+    # of 64 keys fill key tiles 0 (keys 0-191) and 1 (192-383); frame 5 (keys 320-383) lies in
+    # the second half-row of tile 1 only, so with frames = (5,) one warp of each pair alone sees
+    # the jump and the pair's reducing barrier must carry the decision to its partner.
     from paper_2607_00712_gb300 import synth
-    st = Step(8, P=64, H=2, d=64, n_past=6, n_chunk_frames=2, capacity=6)
+    st = Step(8, P=64, H=2, d=d, n_past=6, n_chunk_frames=2, capacity=6)
     P = st.P
-    for f in (4, 5):
+    for f in frames:
         blk = synth.bf16_round(st.s.k_hist[f * P:(f + 1) * P] * np.float32(boost))
         st.s.k_hist[f * P:(f + 1) * P] = blk
         st.k_hist_res[f * P:(f + 1) * P] = blk
