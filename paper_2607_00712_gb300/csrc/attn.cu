@@ -342,26 +342,85 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         tc_commit(b.s_full0 + 8 * (j & 1));   // also tells the TMA thread that K_j has been read
         return true;
       };
-      if (ok) ok = issue_s(0);
-      if (ok && n_tiles > 1) ok = issue_s(1);
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const int vs = j % C::VST;
-        if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
-        tr(j, 3);
-        if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
-        tr(j, 11);
-        tc_fence_after();
-        const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
-        const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
+      if constexpr (!QK8 && C::KST == 2 && C::VST == 2) {
+        // The production shape.  A UMMA stream issues at the full tensor rate only when the
+        // issuing thread has nothing but the instructions themselves to execute between them:
+        // with the loop unrolled by two, the K/V stage and S buffer of each half are known at
+        // compile time and every descriptor is built once, before the loop (measured in
+        // isolation: 77 cycles per UMMA of this tile mix, the pipe's own rate, against 94-108
+        // with the descriptors rebuilt per tile).
+        uint64_t dq[HD / 16], dk[2][HD / 16], dv[2][BN / 16];
 #pragma unroll
-        for (int k = 0; k < BN / 16; ++k) {
-          umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::KBOX, 1024), C::IDESC_PV,
-                  (j > 0 || k > 0) ? 1u : 0u);
+        for (int k = 0; k < HD / 16; ++k) dq[k] = sw128_desc(sQ + (k >> 2) * C::QBOX + (k & 3) * 32, 16, 1024);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+          for (int k = 0; k < HD / 16; ++k)
+            dk[h][k] = sw128_desc(sbase + C::OFF_K + h * C::K_TILE + (k >> 2) * C::KBOX + (k & 3) * 32, 16, 1024);
+#pragma unroll
+          for (int k = 0; k < BN / 16; ++k)
+            dv[h][k] = sw128_desc(sbase + C::OFF_V + h * C::V_TILE + k * 2048, C::KBOX, 1024);
         }
-        tc_commit(b.v_empty0 + 8 * vs);   // V_j read, and O holds tiles 0..j
-        tr(j, 4);
-        if (j + 2 < n_tiles) ok = issue_s(j + 2);
-        tr(j, 5);
+        auto s_tile = [&](int j, int h) -> bool {   // S_j into buffer h = j & 1 from K stage h
+          if (!mbar_wait(b.k_full0 + 8 * h, (j >> 1) & 1, wc, 4, j)) return false;
+          if (j > 0) tr(j, 15);   // K_j landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
+          tc_fence_after();
+          const uint32_t d = tmem + C::COL_S0 + h * BN;
+#pragma unroll
+          for (int k = 0; k < HD / 16; ++k) umma_ss(d, dq[k], dk[h][k], C::IDESC_QK, k > 0 ? 1u : 0u);
+          tc_commit(b.s_full0 + 8 * h);   // also tells the TMA thread that K_j has been read
+          return true;
+        };
+        if (ok) ok = s_tile(0, 0);
+        if (ok && n_tiles > 1) ok = s_tile(1, 1);
+        for (int j0 = 0; ok && j0 < n_tiles; j0 += 2) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int j = j0 + h;
+            if (!ok || j >= n_tiles) break;
+            if (!mbar_wait(b.p_full0 + 8 * h, (j >> 1) & 1, wc, 5, j)) {
+              ok = false;
+              break;
+            }
+            tr(j, 3);
+            if (!mbar_wait(b.v_full0 + 8 * h, (j >> 1) & 1, wc, 6, j)) {
+              ok = false;
+              break;
+            }
+            tr(j, 11);
+            tc_fence_after();
+            const uint32_t a = tmem + C::COL_S0 + h * BN;   // P_j, packed bf16, aliases S_j
+#pragma unroll
+            for (int k = 0; k < BN / 16; ++k)
+              umma_ts(tmem + C::COL_O, a + 8 * k, dv[h][k], C::IDESC_PV, (j > 0 || k > 0) ? 1u : 0u);
+            tc_commit(b.v_empty0 + 8 * h);   // V_j read, and O holds tiles 0..j
+            tr(j, 4);
+            if (j + 2 < n_tiles) ok = s_tile(j + 2, h);
+            tr(j, 5);
+          }
+        }
+      } else {
+        if (ok) ok = issue_s(0);
+        if (ok && n_tiles > 1) ok = issue_s(1);
+        for (int j = 0; ok && j < n_tiles; ++j) {
+          const int vs = j % C::VST;
+          if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
+          tr(j, 3);
+          if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
+          tr(j, 11);
+          tc_fence_after();
+          const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
+          const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
+#pragma unroll
+          for (int k = 0; k < BN / 16; ++k) {
+            umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::KBOX, 1024), C::IDESC_PV,
+                    (j > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit(b.v_empty0 + 8 * vs);   // V_j read, and O holds tiles 0..j
+          tr(j, 4);
+          if (j + 2 < n_tiles) ok = issue_s(j + 2);
+          tr(j, 5);
+        }
       }
       // All UMMAs must have finished before TMEM is released.
       tc_commit(b.drain);
