@@ -818,7 +818,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--no-configs", dest="configs", action="store_false",
                     help="skip the rollout and warmup-to-transition workloads in the extras")
-    ap.add_argument("--cpu-sample-rows", type=int, default=1024)
+    ap.add_argument("--cpu-sample-rows", type=int, default=1536)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--watchdog", type=float, default=300.0, help="dump Python stacks after this many s")
     args = ap.parse_args()
