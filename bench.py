@@ -78,6 +78,19 @@ def peaks():
     return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
 
 
+def roofline_entry(model, achieved, pk):
+    """The roofline object of the F-layer attention launch: achieved TFLOP/s against the measured
+    dense bf16 peak; DRAM traffic per launch only while the kernel source and the model shape are
+    those the ncu counters were taken on."""
+    traffic = None
+    if ATTN_TRAFFIC["model"] == model and attn_source_sha() == ATTN_TRAFFIC["source_sha256_16"]:
+        traffic = ATTN_TRAFFIC["bytes"]
+    return dict(bound="tensor", achieved=round(achieved, 2), peak=pk["bf16"], unit="TFLOP/s",
+                frac=round(achieved / pk["bf16"], 4), traffic=traffic, traffic_unit="bytes per launch",
+                kernel="attn_kernel<128> (F-layer launch)", peak_source=pk["source"] + " burst bf16",
+                frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
+
+
 def attn_flops(nq, nk, d, H):
     return 4.0 * nq * nk * d * H
 
@@ -339,14 +352,7 @@ def run_ours(args, rank, world, local_rank):
         for k_, v_ in list(m.items()):
             if isinstance(v_, float):
                 m[k_] = round(v_, 4)
-    achieved = modes["full"]["tflops"]
-    traffic = None
-    if ATTN_TRAFFIC["model"] == args.model and attn_source_sha() == ATTN_TRAFFIC["source_sha256_16"]:
-        traffic = ATTN_TRAFFIC["bytes"]
-    roofline = dict(bound="tensor", achieved=round(achieved, 2), peak=pk["bf16"], unit="TFLOP/s",
-                    frac=round(achieved / pk["bf16"], 4), traffic=traffic, traffic_unit="bytes per launch",
-                    kernel="attn_kernel<128> (F-layer launch)", peak_source=pk["source"] + " burst bf16",
-                    frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
+    roofline = roofline_entry(args.model, modes["full"]["tflops"], pk)
 
     log(f"[bench] timed steps done at {time.perf_counter() - t_start:.1f} s")
     extras = run_extras(r, wl, device)

@@ -74,3 +74,17 @@ def test_clock_rejection_rule():
     assert bench.clock_rejected(dict(ok, reasons=["sw_thermal_slowdown", "sw_power_cap"]))
     assert bench.clock_rejected(dict(ok, sm_mhz=1400.0))              # stuck low, no reason
     assert not bench.clock_rejected(dict(ok, sm_mhz=1400.0, reasons=["sw_power_cap"]))
+
+
+def test_roofline_traffic_only_for_the_captured_source_and_shape(monkeypatch):
+    import bench
+    pk = dict(bf16=2000.0, bf16_sustained=1600.0, source="measured")
+    r = bench.roofline_entry("1.3b", 1500.0, pk)
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert r["frac"] == 0.75 and r["frac_of_sustained"] == round(1500 / 1600, 4)
+    captured = bench.ATTN_TRAFFIC["source_sha256_16"] == bench.attn_source_sha()
+    assert r["traffic"] == (bench.ATTN_TRAFFIC["bytes"] if captured else None)
+    # another model shape, or a changed kernel source: no traffic figure
+    assert bench.roofline_entry("14b", 1500.0, pk)["traffic"] is None
+    monkeypatch.setattr(bench, "attn_source_sha", lambda: "0" * 16)
+    assert bench.roofline_entry("1.3b", 1500.0, pk)["traffic"] is None
