@@ -73,7 +73,12 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
         torch.cuda.synchronize()
     finally:
         abi.ispa_debug_set_trace(None, 0)
-    t = buf.view(n_tiles, SLOTS).cpu().numpy().astype("int64")
+    return summarise(buf.view(n_tiles, SLOTS).cpu().numpy().astype("int64"))
+
+
+def summarise(t) -> dict:
+    """Medians of the per-tile intervals over the middle tiles, and the first CTA's fill and
+    drain, from the event array t[tile, slot] (clock64 values; 0 where nothing was recorded)."""
     n = int((t[:, 3] != 0).sum())
     J = list(range(10, n - 10)) if n > 30 else list(range(3, max(n - 4, 4)))
 
@@ -96,6 +101,9 @@ def run(model: str = "1.3b", mode: str = "full", frames: int = 18, warmup: int =
         "softmax w0: exp loop done -> P_j arrived": lambda j: t[j, 2] - t[j, 10],
         "softmax w0: S_j seen -> P_j arrived": lambda j: t[j, 2] - t[j, 0],
         "softmax w0: P_j arrived -> S_j+1 seen (waiting for S)": lambda j: t[j + 1, 0] - t[j, 2],
+        # one clock: the chain PV_j -> S_j+2 with both hand-offs; the period is about half of this
+        # plus half of the softmax's own time per tile
+        "softmax w0: P_j arrived -> S_j+2 seen (UMMA chain)": lambda j: t[j + 2, 0] - t[j, 2],
         "spread of S_j seen over the 8 softmax warps": lambda j: max(t[j, 24 + w] for w in range(8)) - min(
             t[j, 24 + w] for w in range(8)),
         "last softmax warp's P_j arrival -> UMMA sees P_j (two clocks)": lambda j: t[j, 3] - last_arrive(j),
