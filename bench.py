@@ -69,6 +69,11 @@ def attn_source_sha():
     return hashlib.sha256(src).hexdigest()[:16]
 
 
+# GB300 datasheet dense (no 2:4 sparsity) bf16 tensor rate per GPU: 2.25 PFLOP/s.  Reported
+# beside the measured cuBLAS peak so that either reading of "% of dense bf16 peak" can be taken.
+NOMINAL_BF16_TFLOPS = 2250.0
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -88,7 +93,21 @@ def roofline_entry(model, achieved, pk):
     return dict(bound="tensor", achieved=round(achieved, 2), peak=pk["bf16"], unit="TFLOP/s",
                 frac=round(achieved / pk["bf16"], 4), traffic=traffic, traffic_unit="bytes per launch",
                 kernel="attn_kernel<128> (F-layer launch)", peak_source=pk["source"] + " burst bf16",
-                frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None)
+                frac_of_sustained=round(achieved / pk["bf16_sustained"], 4) if pk["bf16_sustained"] else None,
+                frac_of_nominal=round(achieved / NOMINAL_BF16_TFLOPS, 4), nominal_peak=NOMINAL_BF16_TFLOPS)
+
+
+def ls_flops(D, T):
+    """FLOPs of one LS accumulation: the method's own work (the upper triangles of G = A^T A and
+    S = Delta^T Delta with their diagonals, and all of X = A^T Delta: 2 T (2 D^2 + D)) and the
+    tile work the kernel issues (256 x 256 tiles with whole diagonal tiles; X in two passes and S
+    in three over the bf16 hi/lo split of Delta, or 128 x 128 tiles when D % 256 != 0)."""
+    method = 2.0 * T * (2.0 * D * D + D)
+    tb = 256 if D % 256 == 0 else 128
+    nb = D // tb
+    upper = nb * (nb + 1) // 2
+    tile = (upper + 2 * nb * nb + 3 * upper) * 2.0 * tb * tb * T
+    return method, tile
 
 
 def attn_flops(nq, nk, d, H):
@@ -143,7 +162,7 @@ class ClockSampler:
         for ln in self.proc.stdout:
             self.lines.append(ln.strip())
 
-    def stop(self):
+    def stop(self, t0: float = 0.0, t1: float = 0.0):
         if self.proc is None:
             return None
         self.proc.terminate()
@@ -170,6 +189,80 @@ class ClockSampler:
         if not sm:
             return None
         return dict(sm_mhz=statistics.median(sm), sm_max_mhz=max(mx), reasons=sorted(reasons), samples=len(sm))
+
+
+class NvmlSampler:
+    """SM clock, power and clock-event reasons read through NVML (read-only queries) every
+    `period` seconds on a thread, so that a timed region of a few tens of ms still holds several
+    samples.  stop() summarises the samples taken inside [t0, t1] (host clock), the window the
+    caller marks as under load.  Raises OSError if NVML cannot be loaded."""
+    # nvmlClocksEventReasons bits
+    BITS = {"sw_power_cap": 0x4, "hw_slowdown": 0x8, "sw_thermal_slowdown": 0x20, "hw_thermal_slowdown": 0x40}
+
+    def __init__(self, gpu: str | int, period: float = 0.004):
+        import ctypes
+        self.ct = ctypes
+        self.nv = ctypes.CDLL("libnvidia-ml.so.1")
+        if self.nv.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        self.h = ctypes.c_void_p()
+        if isinstance(gpu, str) and gpu.startswith(("GPU-", "MIG-")):
+            rc = self.nv.nvmlDeviceGetHandleByUUID(gpu.encode(), ctypes.byref(self.h))
+        else:
+            rc = self.nv.nvmlDeviceGetHandleByIndex_v2(int(gpu), ctypes.byref(self.h))
+        if rc != 0:
+            raise OSError(f"no NVML handle for GPU {gpu}")
+        fn = getattr(self.nv, "nvmlDeviceGetCurrentClocksEventReasons", None)
+        self.reasons_fn = fn or self.nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        self.period = period
+        self.samples: list[tuple[float, int, int, int, int]] = []
+        self.run = False
+        self.t = None
+
+    def _one(self):
+        ct = self.ct
+        sm, mx, mw = ct.c_uint(), ct.c_uint(), ct.c_uint()
+        mask = ct.c_ulonglong()
+        if self.nv.nvmlDeviceGetClockInfo(self.h, 1, ct.byref(sm)) != 0:       # NVML_CLOCK_SM
+            return
+        self.nv.nvmlDeviceGetMaxClockInfo(self.h, 1, ct.byref(mx))
+        self.nv.nvmlDeviceGetPowerUsage(self.h, ct.byref(mw))
+        self.reasons_fn(self.h, ct.byref(mask))
+        self.samples.append((time.perf_counter(), sm.value, mx.value, mw.value, mask.value))
+
+    def _loop(self):
+        while self.run:
+            self._one()
+            time.sleep(self.period)
+
+    def start(self):
+        self.run = True
+        self.t = threading.Thread(target=self._loop, daemon=True)
+        self.t.start()
+
+    def stop(self, t0: float, t1: float):
+        self.run = False
+        if self.t:
+            self.t.join(timeout=2)
+        inside = [x for x in self.samples if t0 <= x[0] <= t1]
+        if not inside:
+            return None
+        reasons = sorted(n for n, b in self.BITS.items() if any(x[4] & b for x in inside))
+        return dict(sm_mhz=statistics.median(x[1] for x in inside), sm_max_mhz=max(x[2] for x in inside),
+                    reasons=reasons, samples=len(inside), power_w_max=round(max(x[3] for x in inside) / 1e3, 1),
+                    source=f"NVML every {self.period * 1e3:.0f} ms inside the timed region")
+
+
+def make_sampler(local_rank: int):
+    """NVML sampler for this rank's GPU, else the nvidia-smi one."""
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    parts = [p.strip() for p in vis.split(",") if p.strip()]
+    gpu = parts[local_rank] if local_rank < len(parts) and not parts[local_rank].isdigit() else \
+        physical_gpu_index(local_rank)
+    try:
+        return NvmlSampler(gpu)
+    except (OSError, AttributeError):
+        return ClockSampler(physical_gpu_index(local_rank))
 
 
 def physical_gpu_index(local_rank: int) -> int:
@@ -266,6 +359,84 @@ class StepRunner:
         rec(5)
 
 
+def timed_steps(r, steps, device, flush, rank, world, local_rank):
+    """Time `steps` chunk steps of runner r: CUDA events between the calls of every step, L2
+    flushed before each step outside its events, a barrier and a device synchronisation on
+    both sides, clocks sampled inside the region.  Returns (segment ms [steps, 5], wall s,
+    clocks); a region whose clocks the timing rules reject is measured once more."""
+    import torch
+    abi = r.abi
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
+
+    def once():
+        sampler = make_sampler(local_rank) if rank == 0 else None
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(device)
+        if sampler:
+            sampler.start()
+            time.sleep(0.05)
+        t0 = time.perf_counter()
+        for k in range(steps):
+            flush.fill_(float(k))          # L2 flush, outside the step's events
+            r.step(evs[k])
+        torch.cuda.synchronize(device)
+        t1 = time.perf_counter()
+        if world > 1:
+            torch.distributed.barrier()
+        clocks = sampler.stop(t0, t1) if sampler else None
+        st, code = abi.ispa_last_device_error()
+        if st != abi.ISPA_OK:
+            raise RuntimeError(f"device error in timed region: {code}")
+        return t1 - t0, clocks
+
+    wall, clocks = once()
+    # A timed region that saw a hardware or thermal slowdown, or SM clocks well below their
+    # maximum with no reason given (a clock lock left by someone else), is measured once more.
+    again = int(clock_rejected(clocks))
+    if world > 1:
+        t = torch.tensor([again], device=device)
+        torch.distributed.broadcast(t, 0)
+        again = int(t.item())
+    if again:
+        log(f"[bench] clocks {clocks}: measuring the timed region once more")
+        first = clocks
+        wall, clocks = once()
+        if clocks is not None:
+            clocks = dict(clocks, remeasured=True, first_attempt=first)
+    seg = np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(5)] for k in range(steps)])
+    return seg, wall, clocks
+
+
+def modes_of(seg, wl, pk):
+    """Per-call means of the timed steps with their rates: attention TFLOP/s (and fraction of the
+    measured dense bf16 peak), LS accumulate method-work and tile-work TFLOP/s, append GB/s."""
+    mean = seg.mean(axis=0)
+    ls_method, ls_tile = ls_flops(wl["D"], wl["nq"])
+    app_bytes = 3 * 2 * 2 * wl["nq"] * wl["D"] * 2
+
+    def attn(ms, fl, nk):
+        tf = fl / (ms * 1e-3) / 1e12
+        return dict(ms=ms, tflops=tf, frac=tf / pk["bf16"], nk=nk)
+
+    modes = dict(
+        full=attn(mean[0], wl["flops_full"], wl["nk_full"]),
+        local=attn(mean[1], wl["flops_local"], wl["nk_local"]),
+        dual=attn(mean[2], wl["flops_dual"], wl["nk_full"]),
+        ls_accumulate=dict(ms=mean[3], method_gflop=ls_method / 1e9,
+                           method_tflops=ls_method / (mean[3] * 1e-3) / 1e12,
+                           method_frac=ls_method / (mean[3] * 1e-3) / 1e12 / pk["bf16"],
+                           tile_tflops=ls_tile / (mean[3] * 1e-3) / 1e12),
+        kv_append=dict(ms=mean[4], gbs=app_bytes / (mean[4] * 1e-3) / 1e9,
+                       frac=app_bytes / (mean[4] * 1e-3) / 1e9 / pk["hbm"]),
+    )
+    for m in modes.values():
+        for k_, v_ in list(m.items()):
+            if isinstance(v_, float):
+                m[k_] = round(v_, 4)
+    return modes
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     device = torch.device("cuda", local_rank)
@@ -291,46 +462,7 @@ def run_ours(args, rank, world, local_rank):
     if st != abi.ISPA_OK:
         raise RuntimeError(f"device error after warmup: {code}")
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
-
-    def timed_run():
-        sampler = ClockSampler(physical_gpu_index(local_rank)) if rank == 0 else None
-        if world > 1:
-            torch.distributed.barrier()
-        torch.cuda.synchronize(device)
-        if sampler:
-            sampler.start()
-            time.sleep(0.3)
-        t0 = time.perf_counter()
-        for k in range(args.steps):
-            flush.fill_(float(k))          # L2 flush, outside the step's events
-            r.step(evs[k])
-        torch.cuda.synchronize(device)
-        wall = time.perf_counter() - t0
-        if world > 1:
-            torch.distributed.barrier()
-        clocks = sampler.stop() if sampler else None
-        st, code = abi.ispa_last_device_error()
-        if st != abi.ISPA_OK:
-            raise RuntimeError(f"device error in timed region: {code}")
-        return wall, clocks
-
-    wall, clocks = timed_run()
-    # A timed region that saw a hardware or thermal slowdown, or SM clocks well below their
-    # maximum with no reason given (a clock lock left by someone else), is measured once more.
-    again = int(clock_rejected(clocks))
-    if world > 1:
-        t = torch.tensor([again], device=device)
-        torch.distributed.broadcast(t, 0)
-        again = int(t.item())
-    if again:
-        log(f"[bench] clocks {clocks}: measuring the timed region once more")
-        first = clocks
-        wall, clocks = timed_run()
-        if clocks is not None:
-            clocks = dict(clocks, remeasured=True, first_attempt=first)
-
-    seg = np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(5)] for k in range(args.steps)])
+    seg, wall, clocks = timed_steps(r, args.steps, device, flush, rank, world, local_rank)
     step_ms = seg.sum(axis=1)
     total_ms = float(step_ms.sum())
     if world > 1:
@@ -340,19 +472,13 @@ def run_ours(args, rank, world, local_rank):
     flops_step = wl["flops_full"] + wl["flops_local"] + wl["flops_dual"]
     ms_per_step = total_ms / args.steps
     value = world * flops_step / (ms_per_step * 1e-3) / 1e12
-    mean = seg.mean(axis=0)
-    modes = dict(
-        full=dict(ms=mean[0], tflops=wl["flops_full"] / (mean[0] * 1e-3) / 1e12, nk=wl["nk_full"]),
-        local=dict(ms=mean[1], tflops=wl["flops_local"] / (mean[1] * 1e-3) / 1e12, nk=wl["nk_local"]),
-        dual=dict(ms=mean[2], tflops=wl["flops_dual"] / (mean[2] * 1e-3) / 1e12, nk=wl["nk_full"]),
-        ls_accumulate=dict(ms=mean[3]),
-        kv_append=dict(ms=mean[4], gbs=3 * 2 * 2 * wl["nq"] * wl["D"] * 2 / (mean[4] * 1e-3) / 1e9),
-    )
-    for m in modes.values():
-        for k_, v_ in list(m.items()):
-            if isinstance(v_, float):
-                m[k_] = round(v_, 4)
+    modes = modes_of(seg, wl, pk)
     roofline = roofline_entry(args.model, modes["full"]["tflops"], pk)
+    # the F-layer's tensor work per SM clock: independent of the clock the peak was measured at
+    if clocks and clocks.get("sm_mhz"):
+        roofline["flop_per_sm_cycle"] = round(wl["flops_full"] / (modes["full"]["ms"] * 1e-3) /
+                                              (clocks["sm_mhz"] * 1e6) / torch.cuda.get_device_properties(
+                                                  device).multi_processor_count, 1)
 
     log(f"[bench] timed steps done at {time.perf_counter() - t_start:.1f} s")
     extras = run_extras(r, wl, device)
@@ -363,6 +489,16 @@ def run_ours(args, rank, world, local_rank):
         log(f"[bench] rollout and warmup configs done at {time.perf_counter() - t_start:.1f} s")
     e2e = run_e2e(r, args, device, flops_step, world)
     log(f"[bench] e2e done at {time.perf_counter() - t_start:.1f} s")
+    launches_per_step = r.launches_per_step
+    del r
+    torch.cuda.empty_cache()
+
+    shapes = {}
+    for other in args.shapes:
+        if other == args.model:
+            continue
+        shapes[other] = run_shape(other, args, device, flush, rank, world, local_rank, pk)
+        log(f"[bench] {other} shape done at {time.perf_counter() - t_start:.1f} s")
 
     result = dict(metric=METRIC, value=round(value, 3), unit=UNIT, n_gpus=world, steps=args.steps,
                   warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
@@ -371,13 +507,41 @@ def run_ours(args, rank, world, local_rank):
                               heads=wl["H"], head_dim=wl["d"], tokens_per_frame=wl["P"], n_q=wl["nq"],
                               f_ring_frames=wl["F"], window_frames=wl["W"], parallelism=f"replicas x{world}",
                               l2="flushed between steps (256 MB write outside timed events)"),
-                  modes=modes, roofline=roofline, e2e=e2e, extras=extras,
-                  gpu_launches=r.launches_per_step * args.steps, clocks=clocks,
+                  modes=modes, roofline=roofline, e2e=e2e, shapes=shapes, extras=extras,
+                  gpu_launches=launches_per_step * args.steps, clocks=clocks,
                   wall_s=round(wall, 3))
     if rank == 0:
         if args.cpu_baseline:
             result["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_rows)
         print(json.dumps(result), flush=True)
+
+
+def run_shape(model, args, device, flush, rank, world, local_rank, pk):
+    """The same chunk step at another model shape, measured exactly like the headline one (same
+    steps, L2 flushed outside the events, clocks sampled), with its own roofline entry and, unless
+    --no-configs, that shape's rollout and warmup-to-transition workloads."""
+    import torch
+    wl = workload(model)
+    r = StepRunner(wl, device, seed=1)
+    for _ in range(args.warmup):
+        r.step()
+    torch.cuda.synchronize(device)
+    seg, wall, clocks = timed_steps(r, args.steps, device, flush, rank, world, local_rank)
+    ms = float(seg.sum(axis=1).mean())
+    flops_step = wl["flops_full"] + wl["flops_local"] + wl["flops_dual"]
+    modes = modes_of(seg, wl, pk)
+    out = dict(workload=f"ISPA chunk step, {model}-shaped layer stack (F + L + dual + LS + append)",
+               heads=wl["H"], head_dim=wl["d"], n_q=wl["nq"], value=round(flops_step / (ms * 1e-3) / 1e12, 3),
+               unit=UNIT, ms_per_step=round(ms, 4), steps=args.steps, modes=modes,
+               roofline=roofline_entry(model, modes["full"]["tflops"], pk), clocks=clocks)
+    del r
+    torch.cuda.empty_cache()
+    if args.configs:
+        out["rollout"] = run_rollout(wl, device, MODEL_LAYERS[model])
+        torch.cuda.empty_cache()
+        out["warmup_to_transition"] = run_warmup(wl, device)
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_extras(r, wl, device, reps=20):
@@ -418,6 +582,27 @@ def run_extras(r, wl, device, reps=20):
     out = dict(decomposed_dual_ms=round(dec, 4), fused_dual_ms=round(t_dual / reps, 4),
                decomposed_merge_ms=round(t_merge / reps, 4),
                merge_share_of_decomposed=round(t_merge / reps / dec, 4))
+    # the decomposed pass's discrepancy from its two stored outputs (HBM-bound: both bf16
+    # [n_q][D] outputs read once, disc written), L2 flushed before every repetition
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=device)
+    disc = torch.empty(nq, dtype=torch.float32, device=device)
+    dsum = torch.zeros(1, dtype=torch.float32, device=device)
+    t_disc = 0.0
+    for i in range(reps + 3):
+        flush.fill_(float(i))
+        ev[0].record(s)
+        abi.ispa_discrepancy(fused, o_loc, nq, D, disc, dsum, s)
+        ev[1].record(s)
+        torch.cuda.synchronize(device)
+        if i >= 3:
+            t_disc += ev[0].elapsed_time(ev[1])
+    t_disc /= reps
+    disc_bytes = 2 * nq * D * 2 + nq * 4
+    pk = peaks()
+    out.update(discrepancy_ms=round(t_disc, 4), discrepancy_gbs=round(disc_bytes / (t_disc * 1e-3) / 1e9, 1),
+               discrepancy_frac_of_hbm=round(disc_bytes / (t_disc * 1e-3) / 1e9 / pk["hbm"], 4),
+               discrepancy_bytes=disc_bytes)
+    del flush
     # closed-form solve of the accumulated state (once per transition)
     from paper_2607_00712_gb300 import synth
     W = torch.from_numpy(synth.make_weight(1, D, D)).to(device)
@@ -821,6 +1006,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--model", choices=sorted(MODELS), default="1.3b")
+    ap.add_argument("--shapes", default="1.3b,14b",
+                    help="model shapes measured after the headline one (comma list; the headline is --model)")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--no-configs", dest="configs", action="store_false",
                     help="skip the rollout and warmup-to-transition workloads in the extras")
@@ -828,6 +1015,10 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--watchdog", type=float, default=300.0, help="dump Python stacks after this many s")
     args = ap.parse_args()
+    args.shapes = [x for x in args.shapes.split(",") if x]
+    for x in args.shapes:
+        if x not in MODELS:
+            ap.error(f"unknown shape {x}")
     import faulthandler
     faulthandler.dump_traceback_later(args.watchdog, exit=False)
     rank = int(os.environ.get("RANK", "0"))

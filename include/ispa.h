@@ -214,6 +214,12 @@ ISPA_API ispa_status ispa_debug_set_trace(uint64_t* buf, int32_t n_tiles);
  * Nothing faults: the missing load simply never arrives.  -1 turns it off (the default). */
 ISPA_API ispa_status ispa_debug_drop_k_tile(int32_t tile);
 
+/* Debug aid for ispa_attn_dual_static: the device address of its scratch array in the
+ * calling thread's current CUDA context (looked up and cached exactly as that entry point
+ * does), the context's process-unique id, and how many address lookups the library has
+ * made so far.  Launches nothing and allocates nothing.  The paper has no counterpart. */
+ISPA_API ispa_status ispa_debug_static_scratch(void** addr, uint64_t* context_id, uint32_t* lookups);
+
 /* Bytes of one ring's K and V buffers together: H * cap * P * d * (2 + 2), or
  * * (1 + 2) with e4m3 keys. */
 ISPA_API size_t ispa_ring_bytes(const ispa_kv_ring* ring);
@@ -341,8 +347,12 @@ ISPA_API ispa_status ispa_attn_dual_ex(const ispa_kv_ring* ring, ispa_window win
  *     GPU that loads it until the process exits; num_heads * n_q must not
  *     exceed ISPA_DUAL_STATIC_MAX_PARTIALS, else ISPA_ERR_WORKSPACE is returned
  *     and nothing is enqueued.
- *   - The first call on a device looks up the array's device address (with
- *     that device current); make that first call before any stream capture.
+ *   - The array's device address belongs to one CUDA context.  The first call
+ *     made with a context current (normally the device's primary context)
+ *     looks it up and caches it under that context's process-unique id, so a
+ *     caller's own context, or the primary context re-created after a
+ *     cudaDeviceReset, gets its own lookup.  Make that first call before any
+ *     stream capture.
  *   - Allocates nothing: no cudaMalloc / cudaFree, no allocating library call.
  *   - All calls share the one array, so calls that overlap on the GPU (e.g.
  *     on two streams) race; serialise them.  Each call overwrites every entry
@@ -375,6 +385,21 @@ ISPA_API ispa_status ispa_attn_hist(const ispa_kv_ring* ring, ispa_window win, c
 ISPA_API ispa_status ispa_lse_merge(const void* o_a, const float* lse_a, const void* o_b, const float* lse_b,
                                     int32_t n_q, int32_t num_heads, int32_t head_dim, void* out, float* lse_out,
                                     ispa_stream stream);
+
+/*
+ * Output discrepancy of the warmup pass (Sec. 3.1 phase 1, which monitors the
+ * discrepancy between the global and the local output; the paper gives no formula,
+ * the reading is disc_t = ||A_full,t - A_loc,t||_2 over all D features) from two
+ * stored outputs -- the discrepancy of the decomposed dual pass (ispa_attn_local +
+ * ispa_attn_hist + ispa_lse_merge); ispa_attn_dual takes it inside its own sweep.
+ *   a_full, a_loc : bf16 [n_q][dim], 16-byte aligned, dim a multiple of 8
+ *                   (else ISPA_ERR_UNSUPPORTED)
+ *   disc          : fp32 [n_q] (overwritten)
+ *   disc_sq_sum   : fp32 device scalar, += sum_t disc_t^2 (not reset)
+ * Differences and sums in fp32.  Asynchronous on `stream`.
+ */
+ISPA_API ispa_status ispa_discrepancy(const void* a_full, const void* a_loc, int32_t n_q, int32_t dim, float* disc,
+                                      float* disc_sq_sum, ispa_stream stream);
 
 /* ------------------------------------------------------------ transition */
 

@@ -77,6 +77,7 @@ _SIGS = {
     "ispa_debug_set_heartbeat": (c_int32, [c_void_p, c_int32]),
     "ispa_debug_set_trace": (c_int32, [c_void_p, c_int32]),
     "ispa_debug_drop_k_tile": (c_int32, [c_int32]),
+    "ispa_debug_static_scratch": (c_int32, [POINTER(c_void_p), POINTER(c_uint64), POINTER(c_uint32)]),
     "ispa_ring_bytes": (c_size_t, [POINTER(KVRing)]),
     "ispa_ring_slot": (c_int32, [POINTER(KVRing), c_int64]),
     "ispa_window_resolve": (c_int32, [POINTER(KVRing), Window, POINTER(KeySets)]),
@@ -103,6 +104,7 @@ _SIGS = {
     "ispa_attn_hist": (c_int32, [POINTER(KVRing), Window, c_void_p, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
     "ispa_lse_merge": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p,
                                  c_void_p]),
+    "ispa_discrepancy": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_select_layers": (c_int32, [POINTER(c_double), c_int32, c_int32, POINTER(c_int32)]),
     "ispa_apply_absorption": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p]),
     "ispa_apply_absorption_bf16": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p]),
@@ -207,6 +209,14 @@ def ispa_debug_drop_k_tile(tile: int) -> None:
     _check(lib().ispa_debug_drop_k_tile(tile), "ispa_debug_drop_k_tile")
 
 
+def ispa_debug_static_scratch() -> tuple[int, int, int]:
+    """(device address, context id, lookups so far) of ispa_attn_dual_static's scratch array."""
+    a, c, n = c_void_p(), c_uint64(), c_uint32()
+    _check(lib().ispa_debug_static_scratch(ctypes.byref(a), ctypes.byref(c), ctypes.byref(n)),
+           "ispa_debug_static_scratch")
+    return int(a.value or 0), int(c.value), int(n.value)
+
+
 def ispa_ring_bytes(ring: KVRing) -> int:
     return lib().ispa_ring_bytes(ctypes.byref(ring))
 
@@ -295,6 +305,11 @@ def ispa_lse_merge(o_a, lse_a, o_b, lse_b, n_q: int, num_heads: int, head_dim: i
                    stream=None) -> None:
     _check(lib().ispa_lse_merge(_ptr(o_a), _ptr(lse_a), _ptr(o_b), _ptr(lse_b), n_q, num_heads, head_dim, _ptr(out),
                                 _ptr(lse_out), _stream(stream)), "ispa_lse_merge")
+
+
+def ispa_discrepancy(a_full, a_loc, n_q: int, dim: int, disc, disc_sq_sum, stream=None) -> None:
+    _check(lib().ispa_discrepancy(_ptr(a_full), _ptr(a_loc), n_q, dim, _ptr(disc), _ptr(disc_sq_sum),
+                                  _stream(stream)), "ispa_discrepancy")
 
 
 def ispa_select_layers(eps, k: int) -> list[int]:

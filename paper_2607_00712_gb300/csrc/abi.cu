@@ -23,7 +23,7 @@ static __device__ int g_status[8];  // device error record (DEVERR_* + location)
 namespace {
 
 constexpr uint64_t kDefaultWaitLimitNs = 1000ull * 1000 * 1000;
-uint64_t g_wait_limit = kDefaultWaitLimitNs;
+std::atomic<uint64_t> g_wait_limit{kDefaultWaitLimitNs};
 
 bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -33,25 +33,47 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
 
 // The tensor-map encoder below is a driver-API call.  In a host thread that has not yet made a
 // CUDA runtime call no context is current, and the encoder fails there (the runtime binds a
 // context only for its own calls).  Bind the current device's primary context first, as the
 // runtime would: a no-op when a context is already current.
+CtxGetCurrentFn ctx_get_current_fn();
+CtxGetIdFn ctx_get_id_fn();
+
 void ensure_context() {
-  static CtxGetCurrentFn get = nullptr;
+  const CtxGetCurrentFn get = ctx_get_current_fn();
+  CUcontext c = nullptr;
+  if (get && get(&c) == CUDA_SUCCESS && c) return;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaSetDevice(dev);
+}
+
+CtxGetCurrentFn ctx_get_current_fn() {
+  static CtxGetCurrentFn fn = nullptr;
   static std::once_flag once;
   std::call_once(once, [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      get = reinterpret_cast<CtxGetCurrentFn>(p);
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
   });
-  CUcontext c = nullptr;
-  if (get && get(&c) == CUDA_SUCCESS && c) return;
-  int dev = 0;
-  if (cudaGetDevice(&dev) == cudaSuccess) cudaSetDevice(dev);
+  return fn;
+}
+
+CtxGetIdFn ctx_get_id_fn() {
+  static CtxGetIdFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  return fn;
 }
 
 EncodeTiledFn encode_fn() {
@@ -70,7 +92,7 @@ EncodeTiledFn encode_fn() {
 
 }  // namespace
 
-uint64_t wait_limit_ns() { return g_wait_limit; }
+uint64_t wait_limit_ns() { return g_wait_limit.load(); }
 
 namespace {
 uint32_t* g_hb = nullptr;   // host-mapped heartbeat buffer (device address), debug only
@@ -94,18 +116,42 @@ uint32_t* next_heartbeat_slot(uint32_t kernel_tag) {
   return slot;
 }
 
+bool current_context_id(uint64_t* id) {
+  ensure_context();
+  const CtxGetCurrentFn get = ctx_get_current_fn();
+  const CtxGetIdFn get_id = ctx_get_id_fn();
+  CUcontext c = nullptr;
+  unsigned long long v = 0;
+  if (!get || !get_id || get(&c) != CUDA_SUCCESS || !c || get_id(c, &v) != CUDA_SUCCESS) return false;
+  *id = static_cast<uint64_t>(v);
+  return true;
+}
+
+// The status record's device address belongs to the context it was looked up in: a
+// caller's own (non-primary) context, or the primary context re-created after a
+// cudaDeviceReset, gets its own lookup, keyed on the context's process-unique id.
 int* device_status_ptr() {
-  static std::atomic<int*> ptrs[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  int* cached = ptrs[dev].load(std::memory_order_acquire);
-  if (!cached) {
+  uint64_t ctx = 0;
+  if (!current_context_id(&ctx)) return nullptr;
+  thread_local uint64_t t_ctx = 0;
+  thread_local int* t_ptr = nullptr;
+  if (t_ptr && t_ctx == ctx) return t_ptr;
+  static std::mutex mu;
+  static std::vector<std::pair<uint64_t, int*>> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  int* found = nullptr;
+  for (const auto& e : cache)
+    if (e.first == ctx) found = e.second;
+  if (!found) {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
-    cached = static_cast<int*>(p);
-    ptrs[dev].store(cached, std::memory_order_release);
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess || !p) return nullptr;
+    found = static_cast<int*>(p);
+    if (cache.size() >= 256) cache.erase(cache.begin());
+    cache.emplace_back(ctx, found);
   }
-  return cached;
+  t_ctx = ctx;
+  t_ptr = found;
+  return found;
 }
 
 cudaError_t set_smem_limit_once(const void* func, int bytes) {
@@ -329,7 +375,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   p.causal_p = (flags & ISPA_ATTN_FRAME_CAUSAL) ? P : 0;
   const float sc = scale == 0.f ? 1.f / sqrtf(static_cast<float>(HD)) : scale;
   p.scale_log2 = sc * 1.4426950408889634f;
-  p.wait_limit_ns = g_wait_limit;
+  p.wait_limit_ns = g_wait_limit.load();
   p.out = static_cast<__nv_bfloat16*>(out);
   p.out_loc = static_cast<__nv_bfloat16*>(out_loc);
   p.lse = lse;
@@ -457,9 +503,7 @@ ispa_status ispa_debug_set_heartbeat(uint32_t* counters, int32_t n_slots) {
 }
 
 uint64_t ispa_set_wait_limit_ns(uint64_t ns) {
-  const uint64_t old = g_wait_limit;
-  g_wait_limit = ns == 0 ? kDefaultWaitLimitNs : ns;
-  return old;
+  return g_wait_limit.exchange(ns == 0 ? kDefaultWaitLimitNs : ns);
 }
 
 ispa_status ispa_debug_wait_probe(uint64_t limit_ns, ispa_stream stream) {
@@ -630,7 +674,7 @@ ispa_status ispa_ls_accumulate(ispa_ls_state* st, const void* a_loc, const void*
   if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
   int* status = device_status_ptr();
   if (!status) return ISPA_ERR_CUDA;
-  if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, st->gram, status, g_wait_limit,
+  if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, st->gram, status, g_wait_limit.load(),
                            next_heartbeat_slot(2), stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   st->n_tokens += T;
@@ -679,7 +723,7 @@ ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uin
   if (D % 128 != 0 || D_out % 128 != 0) return ISPA_ERR_UNSUPPORTED;
   int* status = device_status_ptr();
   if (!status) return ISPA_ERR_CUDA;
-  if (launch_w8a8_gemm(a_q, a_scale, w_q, w_scale, static_cast<int32_t>(T), D, D_out, out, status, g_wait_limit,
+  if (launch_w8a8_gemm(a_q, a_scale, w_q, w_scale, static_cast<int32_t>(T), D, D_out, out, status, g_wait_limit.load(),
                        stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   return ISPA_OK;

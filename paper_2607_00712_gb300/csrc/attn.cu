@@ -495,12 +495,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
         }
       }
-      x_sq[half * BM + row] = sq;
+      // A warp that left through the abort path contributes NaN, so a row whose partial sum
+      // is incomplete reaches disc (and the running sum of disc^2) as NaN, never as a value.
+      x_sq[half * BM + row] = live ? sq : __int_as_float(0x7fc00000);
       soft_barrier();
-      if (live && row_ok && half == 0) {
-        if (lse_dst)
+      if (row_ok && half == 0) {
+        if (live && lse_dst)
           lse_dst[static_cast<size_t>(head) * p.n_q + qrow] = (m_run + __log2f(l_row)) * 0.69314718055994531f;
-        if (with_disc) p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = sq + x_sq[BM + row];
+        if (with_disc)
+          p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = x_sq[row] + x_sq[BM + row];
       }
     };
 

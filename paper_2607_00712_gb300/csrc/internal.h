@@ -120,7 +120,10 @@ cudaError_t launch_append_qk8(const int32_t* slots, int32_t n_frames, int32_t P,
                               const float* k_scale, cudaStream_t s);
 
 // ------------------------------------------------------------ misc
-int* device_status_ptr();  // library status word on the current device (nullptr on error)
+int* device_status_ptr();  // library status word in the current context (nullptr on error)
+// Process-unique id of the calling thread's current CUDA context (the device's primary
+// context is bound first when none is current); false if the driver cannot report it.
+bool current_context_id(uint64_t* id);
 bool encode_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                     uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                     uint32_t b2);

@@ -12,38 +12,58 @@
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds it (ISPA_DUAL_STATIC_MAX_PARTIALS floats) until the process
-// exits.  Its device address is looked up once per device, on the first call
-// made with that device current.
+// exits.  Its device address belongs to one CUDA context.  It is looked up
+// once per context -- normally the device's primary context -- on the first
+// call made with that context current, and cached under the context's
+// process-unique id, so a caller's own context, or the primary context that a
+// cudaDeviceReset re-creates, never receives an address from another one.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <mutex>
+#include <utility>
+#include <vector>
 
 #include "../../include/ispa.h"
+#include "internal.h"
 
 namespace {
 
 static __device__ __align__(256) float g_dual_scratch[ISPA_DUAL_STATIC_MAX_PARTIALS];
 
-constexpr int kMaxDevices = 64;
-float* g_scratch_ptr[kMaxDevices] = {};
 std::mutex g_scratch_mu;
+std::vector<std::pair<uint64_t, float*>> g_scratch_ptr;   // (context id, device address)
+std::atomic<uint32_t> g_scratch_lookups{0};
 
-// Device address of g_dual_scratch on the current device (set-up on first use).
-float* scratch_on_current_device() {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+// Device address of g_dual_scratch in the current context (set-up on first use).
+float* scratch_in_current_context(uint64_t* ctx_out = nullptr) {
+  uint64_t ctx = 0;
+  if (!ispa::current_context_id(&ctx)) return nullptr;
+  if (ctx_out) *ctx_out = ctx;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
-    float* ptr = nullptr;
-    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&ptr), g_dual_scratch) != cudaSuccess || !ptr)
-      return nullptr;
-    g_scratch_ptr[dev] = ptr;
-  }
-  return g_scratch_ptr[dev];
+  for (const auto& e : g_scratch_ptr)
+    if (e.first == ctx) return e.second;
+  float* ptr = nullptr;
+  if (cudaGetSymbolAddress(reinterpret_cast<void**>(&ptr), g_dual_scratch) != cudaSuccess || !ptr) return nullptr;
+  g_scratch_lookups.fetch_add(1);
+  if (g_scratch_ptr.size() >= 256) g_scratch_ptr.erase(g_scratch_ptr.begin());
+  g_scratch_ptr.emplace_back(ctx, ptr);
+  return ptr;
 }
 
 }  // namespace
+
+extern "C" ispa_status ispa_debug_static_scratch(void** addr, uint64_t* context_id, uint32_t* lookups) {
+  if (!addr || !context_id || !lookups) return ISPA_ERR_INVALID_ARG;
+  uint64_t ctx = 0;
+  float* p = scratch_in_current_context(&ctx);
+  if (!p) return ISPA_ERR_CUDA;
+  *addr = p;
+  *context_id = ctx;
+  *lookups = g_scratch_lookups.load();
+  return ISPA_OK;
+}
 
 extern "C" ispa_status ispa_attn_dual_static(const ispa_kv_ring* ring, ispa_window win, const void* q,
                                              const void* k_cur, const void* v_cur, int32_t n_q, float scale,
@@ -52,7 +72,7 @@ extern "C" ispa_status ispa_attn_dual_static(const ispa_kv_ring* ring, ispa_wind
   if (!ring || ring->num_heads <= 0 || n_q <= 0) return ISPA_ERR_INVALID_ARG;
   const size_t need = static_cast<size_t>(ring->num_heads) * static_cast<size_t>(n_q);
   if (need > ISPA_DUAL_STATIC_MAX_PARTIALS) return ISPA_ERR_WORKSPACE;
-  float* scratch = scratch_on_current_device();
+  float* scratch = scratch_in_current_context();
   if (!scratch) return ISPA_ERR_CUDA;
   // The attention kernel writes every (head, query) partial of this call before the
   // reduction reads it, so nothing left over from an earlier call is ever used.

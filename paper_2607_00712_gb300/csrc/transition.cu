@@ -105,6 +105,66 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactParams p) {
     dst[i] = src[i];
 }
 
+// Output discrepancy of two stored outputs (Sec. 3.1 phase 1; reading: the L2 norm over all
+// D features): disc[t] = || a_full[t] - a_loc[t] ||_2 with bf16 rows, differences and sums in
+// fp32, and *disc_sq_sum += sum_t disc[t]^2.  HBM-bound: one warp per token row, each lane
+// streaming 16-byte words of both rows with all its loads issued before the arithmetic.
+constexpr int DISC_WARPS = 8;
+constexpr int DISC_UNROLL = 4;
+
+__device__ __forceinline__ float sq_diff8(const uint4 a, const uint4 b) {
+  const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+  float s = 0.f;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float d0 = __uint_as_float(aw[e] << 16) - __uint_as_float(bw[e] << 16);
+    const float d1 = __uint_as_float(aw[e] & 0xFFFF0000u) - __uint_as_float(bw[e] & 0xFFFF0000u);
+    s = fmaf(d0, d0, s);
+    s = fmaf(d1, d1, s);
+  }
+  return s;
+}
+
+__global__ void __launch_bounds__(DISC_WARPS * 32) discrepancy_kernel(const uint4* __restrict__ af,
+                                                                     const uint4* __restrict__ al, int32_t n_rows,
+                                                                     int32_t words, float* __restrict__ disc,
+                                                                     float* __restrict__ disc_sq_sum) {
+  __shared__ float red[DISC_WARPS];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float mine = 0.f;   // lane 0: this warp's rows
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * DISC_WARPS + warp; r < n_rows;
+       r += static_cast<int64_t>(gridDim.x) * DISC_WARPS) {
+    const uint4* f = af + r * words;
+    const uint4* l = al + r * words;
+    float sq = 0.f;
+    for (int w0 = 0; w0 < words; w0 += 32 * DISC_UNROLL) {
+      uint4 a[DISC_UNROLL], b[DISC_UNROLL];
+#pragma unroll
+      for (int u = 0; u < DISC_UNROLL; ++u) {
+        const int w = w0 + u * 32 + lane;
+        a[u] = w < words ? __ldg(f + w) : make_uint4(0, 0, 0, 0);
+        b[u] = w < words ? __ldg(l + w) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < DISC_UNROLL; ++u) sq += sq_diff8(a[u], b[u]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    if (lane == 0) {
+      disc[r] = sqrtf(sq);
+      mine += sq;
+    }
+  }
+  if (lane == 0) red[warp] = mine;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+#pragma unroll
+    for (int i = 0; i < DISC_WARPS; ++i) t += red[i];
+    atomicAdd(disc_sq_sum, t);
+  }
+}
+
 int grid_for(int64_t n, int threads) {
   int64_t b = (n + threads - 1) / threads;
   if (b > 152 * 8) b = 152 * 8;
@@ -137,6 +197,22 @@ ispa_status ispa_lse_merge(const void* o_a, const float* lse_a, const void* o_b,
   lse_merge_kernel<<<grid_for(total, 256), 256, 0, stream>>>(
       static_cast<const uint4*>(o_a), lse_a, static_cast<const uint4*>(o_b), lse_b, n_q, num_heads, wpr,
       static_cast<uint4*>(out), lse_out);
+  return cudaGetLastError() == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
+}
+
+ispa_status ispa_discrepancy(const void* a_full, const void* a_loc, int32_t n_q, int32_t dim, float* disc,
+                             float* disc_sq_sum, ispa_stream stream) {
+  if (n_q <= 0 || dim <= 0 || !disc || !disc_sq_sum) return ISPA_ERR_INVALID_ARG;
+  if (!aligned16(a_full) || !aligned16(a_loc)) return ISPA_ERR_INVALID_ARG;
+  if (dim % 8 != 0) return ISPA_ERR_UNSUPPORTED;
+  int dev = 0, sms = 152;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // one warp per row; at most 8 CTAs of 256 threads per SM are resident
+  int64_t blocks = (static_cast<int64_t>(n_q) + DISC_WARPS - 1) / DISC_WARPS;
+  if (blocks > static_cast<int64_t>(sms) * 8) blocks = static_cast<int64_t>(sms) * 8;
+  discrepancy_kernel<<<static_cast<unsigned>(blocks), DISC_WARPS * 32, 0, stream>>>(
+      static_cast<const uint4*>(a_full), static_cast<const uint4*>(a_loc), n_q, dim / 8, disc, disc_sq_sum);
   return cudaGetLastError() == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
 }
 

@@ -81,9 +81,7 @@ def summarise(t) -> dict:
     drain, from the event array t[tile, slot] (clock64 values; 0 where nothing was recorded)."""
     n = int((t[:, 3] != 0).sum())
     J = list(range(10, n - 10)) if n > 30 else list(range(3, max(n - 4, 4)))
-
-    def med(f):
-        return int(statistics.median(f(j) for j in J))
+    J = [j for j in J if j + 2 < n]   # every row reads tiles j .. j + 2: traced tiles only
 
     last_arrive = lambda j: max(t[j, 16 + w] for w in range(8))  # noqa: E731
     rows = {
@@ -108,8 +106,11 @@ def summarise(t) -> dict:
             t[j, 24 + w] for w in range(8)),
         "last softmax warp's P_j arrival -> UMMA sees P_j (two clocks)": lambda j: t[j, 3] - last_arrive(j),
     }
-    res = {k: med(f) for k, f in rows.items()}
+    # too few traced tiles for a steady-state middle: no interval rows at all
+    res = {k: int(statistics.median(f(j) for j in J)) for k, f in rows.items()} if J else {}
     res["tiles traced"] = n
+    if n == 0:
+        return res
     # fill and drain of the first CTA (one sample each)
     res["CTA: entry -> TMEM allocated"] = int(t[0, 13] - t[0, 12])
     res["CTA: TMEM allocated -> Q landed"] = int(t[0, 14] - t[0, 13])

@@ -19,6 +19,44 @@ def assert_close_attn(got: np.ndarray, want: np.ndarray, what: str = ""):
     return float(err.max()), float(err.mean())
 
 
+def disc_bound(g_full, g_loc, g_disc, o_full, o_loc):
+    """Per-token bound on |disc_gpu - disc_oracle| derived from the outputs themselves.
+
+    disc_gpu,t = ||Gf_t - Gl_t|| is taken in fp32 over the stored bf16 outputs, disc_or,t =
+    ||Of_t - Ol_t|| in fp64 over the exact ones.  By the triangle inequality
+    | ||x|| - ||y|| | <= ||x - y||, so
+        |disc_gpu,t - disc_or,t| <= ||(Gf_t - Of_t) - (Gl_t - Ol_t)|| + fp32 rounding,
+    the rounding of a sum of D squares in chains of at most 64 + 2 + H terms being below
+    1e-5 relative for every shape here (1e-6 absolute covers an exactly-zero discrepancy).
+    """
+    n = g_full.shape[0]
+    e = (np.asarray(g_full, np.float64) - o_full).reshape(n, -1) - \
+        (np.asarray(g_loc, np.float64) - o_loc).reshape(n, -1)
+    return np.linalg.norm(e, axis=1) + 1e-5 * np.asarray(g_disc, np.float64) + 1e-6
+
+
+def assert_disc_close(g_full, g_loc, g_disc, ref, what="", g_disc_sq_sum=None):
+    """The dual pass's discrepancy against the oracle's, row by row and summed.
+
+    ref: the oracle's attn_dual result for the same rows.  Per token the bound is
+    disc_bound; for the sum of squares |sum g^2 - sum o^2| = |sum (g - o)(g + o)| <=
+    sum b_t (g_t + o_t).  g_disc_sq_sum (optional) is the device accumulator of one call
+    over exactly these rows; its fp32 summation adds at most 1e-5 relative.
+    """
+    g = np.asarray(g_disc, np.float64)
+    o = np.asarray(ref["disc"], np.float64)
+    b = disc_bound(g_full, g_loc, g, ref["a_full"], ref["a_loc"])
+    err = np.abs(g - o)
+    bad = np.nonzero(err > b)[0]
+    assert len(bad) == 0, f"{what}: disc off by {err[bad[:4]]} > bound {b[bad[:4]]} at rows {bad[:4]}"
+    sq_bound = float((b * (g + o)).sum())
+    so = float((o * o).sum())
+    assert abs(float((g * g).sum()) - so) <= sq_bound, f"{what}: sum disc^2"
+    if g_disc_sq_sum is not None:
+        assert abs(float(g_disc_sq_sum) - so) <= sq_bound + 1e-5 * so + 1e-6, f"{what}: disc_sq_sum"
+    return float(err.max()), float(b.max())
+
+
 class Step:
     """A chunk step on the device and the matching oracle inputs.
 

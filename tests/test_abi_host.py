@@ -214,6 +214,10 @@ def test_empty_calls_are_argument_errors_without_gpu():
     assert st.n_tokens == 0
     assert L.ispa_quantize_rows_e4m3(16, 0, 128, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 0, 128, 128, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_discrepancy(16, 16, 0, 128, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_discrepancy(16, 16, 4, 0, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_discrepancy(16, 24, 4, 128, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG   # misaligned row
+    assert L.ispa_discrepancy(16, 16, 4, 100, 16, 16, None) == abi.ISPA_ERR_UNSUPPORTED
 
 
 def test_append_of_more_than_sixteen_frames_is_rejected_without_gpu():

@@ -88,3 +88,42 @@ def test_roofline_traffic_only_for_the_captured_source_and_shape(monkeypatch):
     assert bench.roofline_entry("14b", 1500.0, pk)["traffic"] is None
     monkeypatch.setattr(bench, "attn_source_sha", lambda: "0" * 16)
     assert bench.roofline_entry("1.3b", 1500.0, pk)["traffic"] is None
+
+
+def test_ls_flops_method_and_tile_work():
+    # method work 2T(2D^2 + D): 44.2 GFLOP for the 1.3B step (T 4680, D 1536), 490.8 for 14B
+    m, t = bench.ls_flops(1536, 4680)
+    assert abs(m / 1e9 - 44.18) < 0.01
+    # 256 x 256 tiles: 6 x 6 grid, 21 upper tiles; 21 (G) + 2 * 36 (X) + 3 * 21 (S) = 156 tile-passes
+    assert t == 156 * 2.0 * 256 * 256 * 4680
+    m14, _ = bench.ls_flops(5120, 4680)
+    assert abs(m14 / 1e9 - 490.8) < 0.1
+    # a width with no 256 tiling falls back to 128 x 128 tiles
+    _, t384 = bench.ls_flops(384, 10)
+    assert t384 == (6 + 2 * 9 + 3 * 6) * 2.0 * 128 * 128 * 10
+
+
+def test_modes_rates_and_fractions():
+    import numpy as np
+    wl = bench.workload("1.3b")
+    pk = dict(bf16=2000.0, bf16_sustained=1600.0, hbm=7000.0, source="measured")
+    seg = np.array([[0.6, 0.3, 0.62, 0.08, 0.03]] * 4)
+    m = bench.modes_of(seg, wl, pk)
+    assert abs(m["full"]["tflops"] - wl["flops_full"] / 0.6e-3 / 1e12) < 1e-3
+    assert abs(m["full"]["frac"] - m["full"]["tflops"] / 2000.0) < 1e-4
+    assert abs(m["ls_accumulate"]["method_tflops"] - 44.18e9 / 0.08e-3 / 1e12) < 0.5
+    gbs = 3 * 2 * 2 * 4680 * 1536 * 2 / 0.03e-3 / 1e9
+    assert abs(m["kv_append"]["gbs"] - gbs) < 0.01 and abs(m["kv_append"]["frac"] - gbs / 7000.0) < 1e-4
+
+
+def test_nvml_sampler_window_and_reasons():
+    # the summary keeps only samples inside the timed window and maps the reason bits
+    s = bench.NvmlSampler.__new__(bench.NvmlSampler)
+    s.t, s.run, s.period = None, False, 0.004
+    s.samples = [(0.5, 1200, 2070, 100000, 0x1),           # before the region: idle
+                 (1.0, 2070, 2070, 900000, 0x0), (1.01, 2040, 2070, 950000, 0x4),
+                 (1.02, 2070, 2070, 990000, 0x0), (2.0, 1100, 2070, 100000, 0x8)]   # after it
+    c = s.stop(1.0, 1.5)
+    assert c["samples"] == 3 and c["sm_mhz"] == 2070 and c["reasons"] == ["sw_power_cap"]
+    assert c["power_w_max"] == 990.0
+    assert s.stop(5.0, 6.0) is None

@@ -4,7 +4,9 @@ thread never completes; after the wait limit (2 ms here) the CTA raises its abor
 role leaves through its abort path: the softmax warps keep walking every tile through the same
 warp-pair barriers, the A_loc snapshot and the epilogue.  The call must return, report
 ISPA_ERR_TIMEOUT, and leave the context usable: the same call without the drop then matches a
-plain run bit for bit.  The dual pass is run with the drop before and after its A_loc snapshot."""
+plain run bit for bit.  The dual pass is run with the drop before and after its A_loc snapshot;
+its aborted rows report a NaN discrepancy (and the running sum of disc^2 turns NaN) rather than a
+partial or stale one."""
 import numpy as np
 import pytest
 
@@ -43,7 +45,7 @@ def _run(st, mode):
     ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
     abi.ispa_attn_dual(st.ring.c, Window(0, 2), st.q, st.kc, st.vc, n, 0.0, out, out_loc, disc, dsum, None, None,
                        ws, wsb)
-    return [out, out_loc, disc]
+    return [out, out_loc, disc, dsum]
 
 
 @pytest.mark.parametrize("mode,drop", [("full", 3), ("dual", 3), ("dual", 7)])
@@ -58,7 +60,7 @@ def test_attention_timeout_is_reported_and_recoverable(mode, drop):
     old = abi.ispa_set_wait_limit_ns(2_000_000)
     abi.ispa_debug_drop_k_tile(drop)
     try:
-        _run(st, mode)
+        aborted = _run(st, mode)
         torch.cuda.synchronize()
     finally:
         abi.ispa_debug_drop_k_tile(-1)
@@ -66,6 +68,10 @@ def test_attention_timeout_is_reported_and_recoverable(mode, drop):
     st_code, raw = abi.ispa_last_device_error()
     assert st_code == abi.ISPA_ERR_TIMEOUT and raw == 1, (st_code, raw)
     assert abi.ispa_last_device_error()[0] == abi.ISPA_OK   # reading clears it
+    if mode == "dual":
+        # an aborted row's discrepancy partial is NaN: no stale or partial value reaches disc
+        # or the running sum of disc^2
+        assert np.isnan(aborted[2].cpu().numpy()).all() and np.isnan(float(aborted[3].item()))
     again = _host(_run(st, mode))
     assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
     for a, b in zip(plain, again):

@@ -11,7 +11,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
-from gpu_helpers import Step, assert_close_attn  # noqa: E402
+from gpu_helpers import Step, assert_close_attn, assert_disc_close  # noqa: E402
 from oracle import attention as at  # noqa: E402
 from paper_2607_00712_gb300 import abi  # noqa: E402
 from paper_2607_00712_gb300.device import Window, to_f32  # noqa: E402
@@ -79,7 +79,7 @@ def test_causal_ragged_tiles_and_ring_wrap(d):
         r = at.attn_dual(*args, *win, frame_causal=True)
         assert_close_attn(af, r["a_full"], f"causal dual full {win}")
         assert_close_attn(al, r["a_loc"], f"causal dual loc {win}")
-        assert np.abs(disc - r["disc"]).max() <= 2 * 2e-2 * math.sqrt(st.H * st.d)
+        assert_disc_close(af, al, disc, r, f"causal disc {win}")
 
 
 def test_causal_flag_zero_is_the_plain_call():
@@ -115,7 +115,8 @@ def test_causal_config1_sampled_rows():
     o, _ = _full(st, CAUSAL)
     ro, _ = at.attn_full(*args, rows=rows, frame_causal=True)
     assert_close_attn(o[rows], ro, "config1 causal full")
-    af, al, _ = _dual(st, (0, 6), CAUSAL)
+    af, al, disc = _dual(st, (0, 6), CAUSAL)
     r = at.attn_dual(*args, 0, 6, rows=rows, frame_causal=True)
     assert_close_attn(af[rows], r["a_full"], "config1 causal dual full")
     assert_close_attn(al[rows], r["a_loc"], "config1 causal dual loc")
+    assert_disc_close(af[rows], al[rows], disc[rows], r, "config1 causal disc")

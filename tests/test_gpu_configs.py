@@ -2,15 +2,16 @@
 
 Rows of attention are independent, so the fp64 oracle checks sampled query rows of the
 full-size launches exactly.  LS sums are checked on independent synthetic activations
-(full size for hidden 1536, sampled 128x128 blocks for hidden 5120); the solve is checked
-against the oracle at hidden 1536 and through its normal equations at hidden 5120.
+(full size for hidden 1536, sampled 128x128 blocks for hidden 5120); the solve and eps are
+checked against the oracle's at both hidden sizes (at 5120 on a narrow output weight, with
+numpy's Cholesky as the oracle's factorisation step).
 """
 import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")
 
-from gpu_helpers import Step, assert_close_attn  # noqa: E402
+from gpu_helpers import Step, assert_close_attn, assert_disc_close  # noqa: E402
 from oracle import attention as at  # noqa: E402
 from oracle import ls as ols  # noqa: E402
 from paper_2607_00712_gb300 import abi, synth  # noqa: E402
@@ -87,8 +88,11 @@ def test_warmup_dual_step(heads):
     g_loc = to_f32(a_loc).reshape(n, heads, D_HEAD)
     assert_close_attn(g_full[rows], r["a_full"], "warmup a_full")
     assert_close_attn(g_loc[rows], r["a_loc"], "warmup a_loc")
+    g_disc = to_f32(disc)
+    assert_disc_close(g_full[rows], g_loc[rows], g_disc[rows], r, "warmup disc")
+    # extra: self-consistency of disc and of the device sum over all tokens
     d_own = np.sqrt(((g_full.astype(np.float64) - g_loc) ** 2).reshape(n, -1).sum(1))
-    assert np.allclose(to_f32(disc), d_own, rtol=1e-5, atol=1e-5)
+    assert np.allclose(g_disc, d_own, rtol=1e-5, atol=1e-5)
     assert abs(float(dsum.item()) - float((d_own ** 2).sum())) <= 1e-4 * float((d_own ** 2).sum())
 
 
@@ -128,27 +132,52 @@ def test_warmup_ls_hidden1536_full():
     assert abs(eps - eps_ref) <= 1e-3 * abs(eps_ref)
 
 
-def test_warmup_ls_hidden5120_sampled_blocks_and_normal_equations():
-    # Hidden 5120: G/X/S on sampled 128x128 blocks (each computed by the oracle from its own
-    # column slices), and the solve through the normal equations with the oracle's sums.
-    D, T = 5120, 10240
+def _sym_upper(M):
+    """The symmetric matrix whose upper triangle the state maintains."""
+    return np.triu(M) + np.triu(M, 1).T
+
+
+def test_warmup_ls_hidden5120_sums_solve_and_eps():
+    # Hidden 5120 (the 14B shape).  G/X/S on sampled 128x128 blocks against the oracle's sums;
+    # then the solve and eps on a narrow output weight (d_out = 96), both sides from the SAME
+    # accumulated state (the GPU's, read back), so the comparison isolates the solve.
+    D, T, D_OUT, LAM = 5120, 10240, 96, 1e-3
     a, f = synth.make_activations(600, T, D)
     st = _accumulate_gpu(D, [(a, f)])
     G, X, S = st.blocks()
-    a64, d64 = a.astype(np.float64), f.astype(np.float64) - a.astype(np.float64)
+    ref = ols.ls_accumulate(ols.ls_state(D), a, f)
     for (i, j) in [(0, 0), (0, 39), (17, 23), (39, 39), (5, 5)]:
         I, J = slice(128 * i, 128 * i + 128), slice(128 * j, 128 * j + 128)
-        for name, got, want in [("G", G[I, J], a64[:, I].T @ a64[:, J]), ("X", X[I, J], a64[:, I].T @ d64[:, J]),
-                                ("S", S[I, J], d64[:, I].T @ d64[:, J])]:
+        for name, got, want in [("G", G[I, J], ref["G"][I, J]), ("X", X[I, J], ref["X"][I, J]),
+                                ("S", S[I, J], ref["S"][I, J])]:
             assert np.linalg.norm(got - want) / np.linalg.norm(want) <= 1e-3, (name, i, j)
-    W = synth.make_weight(10, D, D)
-    wsb = abi.ispa_ls_solve_workspace_size(D, D)
+    W = synth.make_weight(10, D, D_OUT)
+    wsb = abi.ispa_ls_solve_workspace_size(D, D_OUT)
     ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
-    dW = torch.empty(D, D, dtype=torch.float32, device="cuda")
-    abi.ispa_ls_solve(st.c, torch.from_numpy(W).cuda(), D, 1e-3, dW, ws, wsb)
+    dW = torch.empty(D, D_OUT, dtype=torch.float32, device="cuda")
+    eps = abi.ispa_ls_solve(st.c, torch.from_numpy(W).cuda(), D_OUT, LAM, dW, ws, wsb)
     dWg = to_f32(dW).astype(np.float64)
-    Gref = a64.T @ a64
-    Xref = a64.T @ d64
-    rhs = Xref @ W.astype(np.float64)
-    res = (Gref + 1e-3 * np.eye(D)) @ dWg - rhs
-    assert np.linalg.norm(res) / np.linalg.norm(rhs) <= 1e-3
+    Gs, Ss = _sym_upper(G), _sym_upper(S)
+    dW_or, eps_or = ols.ls_solve(Gs, X, Ss, W, LAM, factor=np.linalg.cholesky)
+    # dW: both solves are fp64 on the same state; the GPU stores dW in fp32 (relative
+    # rounding <= 2^-24 per entry), and fp64 rounding times cond(G + lambda I) (~34 for
+    # T = 2D Gaussian rows) stays far below 1e-6
+    assert np.linalg.norm(dWg - dW_or) <= 1e-6 * np.linalg.norm(dW_or)
+    # normal equations of the GPU's dW: the residual of the exact solution is fp64 noise, so
+    # what remains is |G + lambda I| |round_fp32(dW) - dW| <= 2^-24 |G + lambda I| |dW|
+    M = Gs + LAM * np.eye(D)
+    rhs = X @ W.astype(np.float64)
+    res = np.linalg.norm(M @ dWg - rhs)
+    bound = 2.0 ** -24 * np.linalg.norm(np.abs(M) @ np.abs(dWg)) + 1e-12 * np.linalg.norm(rhs)
+    assert res <= bound, (res, bound)
+    # eps (Eq. 6 through its trace form; Sec. 3.3 ranks layers by it): a difference of large
+    # terms, each formed in fp64 on both sides; allow 1e-9 of the terms' magnitude
+    terms = (abs(np.sum(dW_or * (Gs @ dW_or))) + 2 * abs(np.sum(dW_or * rhs))
+             + abs(np.sum(W.astype(np.float64) * (Ss @ W.astype(np.float64)))))
+    assert abs(eps - eps_or) <= 1e-9 * terms, (eps, eps_or, terms)
+    assert eps_or > 0
+    # end to end: the GPU solve of the GPU sums against the oracle's solve of its own sums,
+    # within what the 1e-3 bound on the sums allows through cond(G + lambda I)
+    dW_e2e, eps_e2e = ols.ls_solve(ref["G"], ref["X"], ref["S"], W, LAM, factor=np.linalg.cholesky)
+    assert np.linalg.norm(dWg - dW_e2e) <= 1e-3 * np.linalg.norm(dW_e2e)
+    assert abs(eps - eps_e2e) <= 1e-3 * abs(eps_e2e)

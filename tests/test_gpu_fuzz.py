@@ -10,7 +10,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
-from gpu_helpers import Step, assert_close_attn  # noqa: E402
+from gpu_helpers import Step, assert_close_attn, assert_disc_close  # noqa: E402
 from oracle import attention as at  # noqa: E402
 from oracle import keysets as ks  # noqa: E402
 from paper_2607_00712_gb300 import abi  # noqa: E402
@@ -85,6 +85,8 @@ def test_random_step(i):
     r = at.attn_dual(*args, *win, frame_causal=c["causal"])
     assert_close_attn(to_f32(a_full).reshape(ro.shape), r["a_full"], f"case {i} dual full {c}")
     assert_close_attn(to_f32(a_loc).reshape(ro.shape), r["a_loc"], f"case {i} dual loc {c}")
+    assert_disc_close(to_f32(a_full).reshape(ro.shape), to_f32(a_loc).reshape(ro.shape), to_f32(disc), r,
+                      f"case {i} disc {c}", float(dsum.item()))
 
     # the paper's two-call decomposition (Eq. 9-12) on the dense chunk
     if not c["causal"]:

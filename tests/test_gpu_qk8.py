@@ -11,7 +11,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
-from gpu_helpers import assert_close_attn  # noqa: E402
+from gpu_helpers import assert_close_attn, assert_disc_close  # noqa: E402
 from oracle import attention as at  # noqa: E402
 from oracle import keysets as ks  # noqa: E402
 from oracle import quant as qt  # noqa: E402
@@ -180,6 +180,8 @@ def test_qk8_dual_matches_oracle():
     assert_close_attn(to_f32(a_full).reshape(r["a_full"].shape), r["a_full"], "qk8 dual full")
     assert_close_attn(to_f32(a_loc).reshape(r["a_loc"].shape), r["a_loc"], "qk8 dual loc")
     got = to_f32(disc)
+    assert_disc_close(to_f32(a_full).reshape(r["a_full"].shape), to_f32(a_loc).reshape(r["a_loc"].shape), got, r,
+                      "qk8 disc", float(dsum.item()))
     own = np.sqrt(((to_f32(a_full).astype(np.float64) - to_f32(a_loc)) ** 2).sum(1))
     assert np.allclose(got, own, rtol=1e-5, atol=1e-6)
 

@@ -5,7 +5,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
-from gpu_helpers import Step, assert_close_attn  # noqa: E402
+from gpu_helpers import Step, assert_close_attn, assert_disc_close  # noqa: E402
 from oracle import attention as at  # noqa: E402
 from oracle import keysets as ks  # noqa: E402
 from paper_2607_00712_gb300 import abi, synth  # noqa: E402
@@ -48,6 +48,15 @@ def test_decomposed_dual_matches_oracle(win):
     r_full, rl_full = at.attn_full(*args)
     assert_close_attn(to_f32(fused).reshape(r_full.shape), r_full, "decomposed A_full")
     assert np.abs(to_f32(lse) - rl_full).max() < 2e-3
+    # the decomposed pass's discrepancy (Sec. 3.1 phase 1) from its two stored outputs
+    disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    abi.ispa_discrepancy(fused, o_loc, st.n_q, st.H * st.d, disc, dsum)
+    torch.cuda.synchronize()
+    r = at.attn_dual(*args, *win)
+    g_full = to_f32(fused).reshape(r_full.shape)
+    g_loc = to_f32(o_loc).reshape(r_full.shape)
+    assert_disc_close(g_full, g_loc, to_f32(disc), r, "decomposed disc", float(dsum.item()))
 
 
 def test_decomposed_dual_empty_history():
@@ -126,3 +135,32 @@ def test_apply_absorption():
     torch.cuda.synchronize()
     exact = Wb.astype(np.float64) + dW.astype(np.float64)
     assert np.all(np.abs(to_f32(Wbt) - exact) <= 2 ** -8 * np.abs(exact) + 1e-30)
+
+
+@pytest.mark.parametrize("n,dim", [(1, 8), (37, 264), (4680, 1536), (1000, 5120)])
+def test_discrepancy_of_stored_outputs(n, dim):
+    # disc_t = ||a_t - b_t||_2 of two bf16 rows (differences of bf16 values are exact in fp32;
+    # the fp32 sums of dim squares stay within 1e-5 relative of the fp64 norms), and the running
+    # sum of disc^2 over two calls; ragged word counts (264 = 33 words) and the model widths
+    a, b = synth.make_activations(400 + n, n, dim)
+    disc = torch.empty(n, dtype=torch.float32, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    ta, tb = bf16_tensor(a), bf16_tensor(b)
+    abi.ispa_discrepancy(ta, tb, n, dim, disc, dsum)
+    abi.ispa_discrepancy(ta, tb, n, dim, disc, dsum)
+    torch.cuda.synchronize()
+    want, want_sq = at.discrepancy(a, b)
+    assert np.allclose(to_f32(disc), want, rtol=1e-5, atol=1e-6)
+    assert abs(float(dsum.item()) - 2 * want_sq) <= 1e-5 * 2 * want_sq
+
+
+def test_discrepancy_rejects_bad_arguments():
+    x = torch.zeros(16, 64, dtype=torch.bfloat16, device="cuda")
+    disc = torch.empty(16, dtype=torch.float32, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    with pytest.raises(abi.IspaError) as e:
+        abi.ispa_discrepancy(x, x, 16, 60, disc, dsum)
+    assert e.value.status == abi.ISPA_ERR_UNSUPPORTED
+    with pytest.raises(abi.IspaError) as e:
+        abi.ispa_discrepancy(x, x, 0, 64, disc, dsum)
+    assert e.value.status == abi.ISPA_ERR_INVALID_ARG

@@ -155,3 +155,18 @@ def test_triangular_solves_against_library():
     B = r.standard_normal((15, 4))
     assert np.allclose(ls.forward_sub(L, B), np.linalg.solve(L, B), atol=1e-12)
     assert np.allclose(ls.back_sub(L.T, B), np.linalg.solve(L.T, B), atol=1e-12)
+
+
+def test_solve_with_library_factor_matches_textbook():
+    # the library Cholesky used at hidden 5120 gives the textbook path's dW and eps
+    r = np.random.default_rng(11)
+    a, f = r.standard_normal((400, 48)), r.standard_normal((400, 48))
+    W = r.standard_normal((48, 7))
+    st = _state(a, f)
+    dW0, e0 = ls.ls_solve(st["G"], st["X"], st["S"], W, 1e-3)
+    dW1, e1 = ls.ls_solve(st["G"], st["X"], st["S"], W, 1e-3, factor=np.linalg.cholesky)
+    assert np.linalg.norm(dW1 - dW0) <= 1e-12 * np.linalg.norm(dW0)
+    assert abs(e1 - e0) <= 1e-10 * abs(e0)
+    # and still satisfies the normal equations to the oracle's bound
+    rhs = st["X"] @ W
+    assert np.linalg.norm((st["G"] + 1e-3 * np.eye(48)) @ dW1 - rhs) / np.linalg.norm(rhs) <= 1e-10

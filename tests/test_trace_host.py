@@ -50,3 +50,14 @@ def test_summarise_recovers_the_planted_intervals():
     assert r["CTA: entry -> TMEM allocated"] == 1400
     assert r["CTA: TMEM allocated -> Q landed"] == 2200
     assert r["CTA: last P seen -> epilogue stored"] == 5000
+
+
+def test_short_traces_report_only_traced_tiles():
+    # 6 tiles: the one middle tile j = 3 has j + 2 = 5 traced, so every row is a real interval
+    r = summarise(_trace(6))
+    assert r["period (UMMA thread sees P_j -> sees P_j+1)"] == PERIOD
+    assert r["softmax w0: P_j arrived -> S_j+2 seen (UMMA chain)"] == 2 * PERIOD - 2150
+    assert r["tiles traced"] == 6
+    # 4 tiles: no middle tile with two traced successors, so no interval row is printed
+    r = summarise(_trace(4))
+    assert "period (UMMA thread sees P_j -> sees P_j+1)" not in r and r["tiles traced"] == 4

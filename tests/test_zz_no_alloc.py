@@ -87,3 +87,49 @@ def test_static_scratch_rejects_oversize_before_launch():
     st = abi.lib().ispa_attn_dual_static(ctypes.byref(r), Window(0, 1), 16, 16, 16, n_q, 0.0, 16, 16, 16, 16,
                                          None, None, None)
     assert st == abi.ISPA_ERR_WORKSPACE
+
+
+_CONTEXT_CHILD = r"""
+import ctypes, sys
+sys.path.insert(0, sys.argv[1])
+from paper_2607_00712_gb300 import abi
+cu = ctypes.CDLL("libcuda.so.1")
+assert cu.cuInit(0) == 0
+a1, c1, n1 = abi.ispa_debug_static_scratch()          # the primary context, bound by the library
+assert a1 != 0
+assert abi.ispa_debug_static_scratch() == (a1, c1, n1)  # cached: no second lookup
+dev = ctypes.c_int()
+assert cu.cuDeviceGet(ctypes.byref(dev), 0) == 0
+ctx = ctypes.c_void_p()
+if not hasattr(cu, "cuCtxCreate_v2") or cu.cuCtxCreate_v2(ctypes.byref(ctx), 0, dev) != 0:
+    print("no-ctx-create")
+    sys.exit(0)
+try:
+    a2, c2, n2 = abi.ispa_debug_static_scratch()       # the caller's own context is current now
+    assert c2 != c1 and n2 == n1 + 1, (c1, c2, n1, n2)
+    assert abi.ispa_debug_static_scratch() == (a2, c2, n2)
+finally:
+    assert cu.cuCtxDestroy_v2(ctx) == 0                 # the primary context is current again
+a3, c3, n3 = abi.ispa_debug_static_scratch()
+assert (a3, c3) == (a1, c1) and n3 == n2, (a1, c1, a3, c3, n2, n3)
+print("ok")
+"""
+
+
+def test_static_scratch_address_is_keyed_on_the_current_context():
+    # A caller that makes its own CUDA context current must not be handed the scratch address
+    # looked up in another context (a kernel given it would fault).  In a child process that
+    # uses only the driver API and the library (no kernel is launched): the primary context's
+    # address is looked up once and reused; a context the caller creates gets a lookup of its
+    # own; once that context is destroyed the primary context's cached entry is used again.
+    # A primary context re-created by cudaDeviceReset carries a new process-unique id too, so
+    # it takes the same path as the created context here.
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _CONTEXT_CHILD, root], capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stdout + r.stderr
+    if "no-ctx-create" in r.stdout:
+        pytest.skip("the driver offers no cuCtxCreate_v2")
+    assert r.stdout.strip().endswith("ok"), r.stdout + r.stderr
