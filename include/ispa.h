@@ -24,6 +24,9 @@
  *     non-OK return of argument validation nothing has been enqueued.
  *   - Kernels never spin without bound: a wait that runs out records a device
  *     error, which ispa_last_device_error() reports as ISPA_ERR_TIMEOUT.
+ *   - The attention kernels launch one CTA per (query tile, head); the CTAs
+ *     that start first take the items of CTAs that have not started yet
+ *     (cluster launch control), so each SM works through a run of items.
  *   - Head dims supported: 64 and 128.  Tokens per frame P >= 1.
  *   - Counts (queries n_q, tokens T, frames n_frames, rows) must be at least
  *     1: an empty call is an argument error (ISPA_ERR_INVALID_ARG) and
@@ -319,6 +322,9 @@ ISPA_API size_t ispa_attn_dual_workspace_size(int32_t num_heads, int32_t n_q);
  *   lse_full, lse_loc : fp32 [num_heads][n_q] or NULL
  *   workspace      : >= ispa_attn_dual_workspace_size bytes
  * An empty history set gives a_full == a_loc bit for bit and disc == 0.
+ * If a device wait runs out (ISPA_ERR_TIMEOUT), the outputs of the call are
+ * undefined and disc_sq_sum becomes NaN: an aborted row contributes a NaN
+ * partial, so a running sum never silently absorbs a partial or stale value.
  */
 ISPA_API ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void* q,
                            const void* k_cur, const void* v_cur, int32_t n_q, float scale,

@@ -91,8 +91,13 @@ struct Cfg {
   static constexpr int X_FLOATS = 2 * 2 * BM;  // [block][half][BM]: pair exchanges and the epilogue
   static constexpr int OFF_FLAG = OFF_X + X_FLOATS * 4;  // pair status [half][quarter] (int)
   static constexpr int OFF_BAR = OFF_FLAG + 32;
-  static constexpr int N_BAR = 1 + KST + 2 * VST + 4 + 1;
-  static constexpr int SMEM = OFF_BAR + N_BAR * 8 + 16;  // + tmem slot / abort flag / spare
+  // q, K stages, V full/empty, S x2, P x2, drain, try_cancel, item mailbox full/empty x2
+  static constexpr int N_BAR = 1 + KST + 2 * VST + 4 + 1 + 1 + 4;
+  static constexpr int OFF_MISC = (OFF_BAR + N_BAR * 8 + 15) / 16 * 16;   // tmem slot, abort flag, spare
+  static constexpr int OFF_CLC = OFF_MISC + 16;          // try_cancel response (16 B)
+  static constexpr int OFF_ITEMS = OFF_CLC + 16;         // item mailbox: 2 slots of (q tile, head)
+  static constexpr int SMEM = OFF_ITEMS + 16;
+  static_assert(OFF_CLC % 16 == 0, "try_cancel response alignment");
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
   static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
@@ -103,7 +108,7 @@ struct Cfg {
 };
 
 struct Bars {
-  uint32_t q_full, k_full0, v_full0, v_empty0, s_full0, p_full0, drain;
+  uint32_t q_full, k_full0, v_full0, v_empty0, s_full0, p_full0, drain, clc, item_full0, item_empty0;
 };
 
 __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& off) {
@@ -174,8 +179,23 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 }  // namespace
 
 // TRACE: the instance launched while a trace buffer is set records the per-tile events of
-// ispa_debug_set_trace; the production instances contain no trace code at all (even an
-// untaken clock64 read constrains instruction scheduling: it cost 6 % here).
+// ispa_debug_set_trace (first work item of CTA (0, 0)); the production instances contain no
+// trace code at all (even an untaken clock64 read constrains instruction scheduling: it cost 6 %
+// here).
+//
+// Work items.  A work item is one (query tile, head); the grid has one CTA per item.  A running
+// CTA takes further items from the CTAs of the grid that have not started yet (cluster launch
+// control try_cancel: a cancelled CTA never runs and its item is done here), so the CTAs that
+// hold the SMs stay resident until no item is left and the SMs that finish first take more
+// items.  Item k of a CTA covers its key tiles g = k * n_tiles + j (j = 0 .. n_tiles - 1): stage
+// rings, S buffers and barrier phases count g, so the TMA and UMMA pipelines run on across item
+// boundaries and the next item's Q, first K/V tiles and first two S tiles overlap this item's
+// last tile and epilogue.  At a boundary the UMMA stream is ... S_n-1 PV_n-2 PV_n-1 S'_0 S'_1
+// PV'_0 ...: the next item's first S tiles reuse the buffers of P_n-2 and P_n-1 after both PVs,
+// and PV'_0 (which overwrites O) follows P'_0, which the softmax warps publish after the
+// epilogue's reads of O.
+// The TMA thread asks for the next item a few tiles before the end of the current one and
+// publishes it (or "none") to the UMMA thread and the softmax warps through a two-slot mailbox.
 template <int HD, bool QK8, bool TRACE>
 __global__ void __launch_bounds__(NTHREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kr,
@@ -196,14 +216,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   float* x_max = reinterpret_cast<float*>(smem + C::OFF_X);  // [block][half][row]
   volatile int* x_flag = reinterpret_cast<volatile int*>(smem + C::OFF_FLAG);   // [half][quarter]
   uint64_t* bar_mem = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_mem + C::N_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* mailbox = reinterpret_cast<volatile int*>(smem + C::OFF_ITEMS);   // [slot][q tile, head]
+  const uint32_t clc_resp = sbase + C::OFF_CLC;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int q_tile = blockIdx.x;
-  const int head = blockIdx.y;
-  const int q0 = q_tile * BM;
 
   Bars b;
   {
@@ -215,6 +234,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     b.s_full0 = b.v_empty0 + 8 * C::VST;
     b.p_full0 = b.s_full0 + 16;
     b.drain = b.p_full0 + 16;
+    b.clc = b.drain + 8;
+    b.item_full0 = b.clc + 8;
+    b.item_empty0 = b.item_full0 + 16;
   }
 
   if (threadIdx.x == 0) {
@@ -229,8 +251,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(b.s_full0 + 8 * i, 1);
       mbar_init(b.p_full0 + 8 * i, N_SOFT);
+      mbar_init(b.item_full0 + 8 * i, 1);
+      mbar_init(b.item_empty0 + 8 * i, 1 + N_SOFT_WARPS);   // the UMMA thread + one lane per softmax warp
     }
     mbar_init(b.drain, 1);
+    mbar_init(b.clc, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -253,8 +278,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const uint32_t tmem = *tmem_slot;
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
   const int n_tiles = p.n_tiles;
-  auto tr = [&](int tile, int ev) {
-    if constexpr (TRACE) trace_event(p.trace, p.trace_tiles, tile, ev);
+  // tile events of the CTA's first item (global tile index = item tile index there)
+  auto tr = [&](int g, int ev) {
+    if constexpr (TRACE) {
+      if (g < n_tiles) trace_event(p.trace, p.trace_tiles, g, ev);
+    }
   };
   if constexpr (TRACE) {
     // once per CTA, in tile 0's spare slots: 12 kernel entry, 13 TMEM allocated
@@ -266,50 +294,121 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       const uint32_t sQ = sbase + C::OFF_Q;
-      mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
-      tma_load_4d(sQ, &tm_q, b.q_full, 0, q0, 0, head);
-      // Loads are issued in the order their stages free up: the UMMA stream is
-      // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so K_t goes out once S_t-2 has completed and
-      // V_{t-1} once PV_{t-1-VST} has; V therefore trails K by one tile.
-      int kseg = 0, koff = 0, vseg = 0, voff = 0;
-      int nk = 0, nv = 0;  // K and V tiles issued
-      for (int t = 0; t <= n_tiles; ++t) {
-        if (t == p.drop_k_tile) break;   // debug: this load never goes out (timeout-path test)
-        if (t < n_tiles) {
-          const bool chunk = p.seg[kseg].src != 0;
-          const int row = p.seg[kseg].start + koff;
+      // item (q tile, head) of the K cursor, and the head of the item before it: V trails K by
+      // at most one tile, so it is on one of the two
+      int kq = static_cast<int>(blockIdx.x), kh = static_cast<int>(blockIdx.y), prev_h = kh;
+      bool can_steal = true;     // no try_cancel has failed yet
+      int n_req = 0, n_resp = 0;  // try_cancel requests issued / responses consumed
+      int nq = 0;                 // Q tiles issued
+      auto request = [&]() {
+        if (!can_steal) return;
+        fence_proxy_async_smem();
+        mbar_arrive_expect_tx(b.clc, 16);
+        clc_try_cancel(clc_resp, b.clc);
+        ++n_req;
+      };
+      auto load_q = [&]() {   // Q of the K cursor's item
+        mbar_arrive_expect_tx(b.q_full, C::Q_TILE);
+        tma_load_4d(sQ, &tm_q, b.q_full, 0, kq * BM, 0, kh);
+        ++nq;
+      };
+      // the request for the item after item k goes out this many K tiles before its end
+      const int req_at = n_tiles > 4 ? n_tiles - 4 : 0;
+      int kk = 0, kj = 0, kseg = 0, koff = 0;   // K cursor: item, tile of the item, segment walk
+      int vk = 0, vj = 0, vseg = 0, voff = 0;   // V cursor
+      int t = 0, tv = 0;                        // global K and V tiles issued
+      bool k_live = true, ok = true;
+      load_q();
+      if (req_at == 0) request();
+      // Loads are issued in the order their stages free up: inside an item the UMMA stream is
+      // S_0 S_1 PV_0 S_2 PV_1 S_3 ..., so K_t goes out once S_t-2 has completed and V_t-1 once
+      // PV_t-1-VST has; V therefore trails K by one tile.
+      auto issue_v = [&]() -> bool {
+        const int vs = tv % C::VST;
+        if (!mbar_wait(b.v_empty0 + 8 * vs, ((tv / C::VST) & 1) ^ 1, wc, 2, tv)) return false;
+        const bool chunk = p.seg[vseg].src != 0;
+        mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::V_TILE);
+        tma_load_4d(sbase + C::OFF_V + vs * C::V_TILE, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0,
+                    p.seg[vseg].start + voff, 0, vk == kk ? kh : prev_h);
+        tr(tv, 7);
+        ++tv;
+        if (++vj == n_tiles) {
+          vj = vseg = voff = 0;
+          ++vk;
+        } else {
+          next_tile(p, vseg, voff);
+        }
+        return true;
+      };
+      while (ok) {
+        if (k_live) {
+          if (kj == 0 && kk > 0) {
+            // item boundary: the previous item's last V first (its PV comes next in the UMMA
+            // stream), then the next item's Q once the previous item's last S has read Q
+            if (tv < t && !issue_v()) break;
+            if (!mbar_wait(b.s_full0 + 8 * ((t - 1) & 1), ((t - 1) >> 1) & 1, wc, 1, t)) break;
+            load_q();
+            if (req_at == 0) request();
+          }
+          if (kj == p.drop_k_tile) break;   // debug: this load never goes out (timeout-path test)
           const int ks = t % C::KST;
           // K_t's stage held K_t-KST; S_t-2 complete means K_t-2 (and every older K) has been
           // read.  S_t cannot complete before K_t lands, so this barrier is never a phase ahead.
           if (t >= 2 && !mbar_wait(b.s_full0 + 8 * ((t - 2) & 1), ((t - 2) >> 1) & 1, wc, 1, t)) break;
+          const bool chunk = p.seg[kseg].src != 0;
           mbar_arrive_expect_tx(b.k_full0 + 8 * ks, C::K_TILE);
-          const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
-          tma_load_4d(sK, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0, row, 0, head);
-          nk = t + 1;
+          tma_load_4d(sbase + C::OFF_K + ks * C::K_TILE, chunk ? &tm_kc : &tm_kr, b.k_full0 + 8 * ks, 0,
+                      p.seg[kseg].start + koff, 0, kh);
           tr(t, 6);
-          next_tile(p, kseg, koff);
+          ++t;
+          if (++kj == req_at && req_at > 0) request();
+          if (kj == n_tiles) {
+            // end of item kk: learn item kk + 1 (a cancelled CTA's item, or none) and post it
+            int nx = -1, ny = -1;
+            if (n_req > n_resp) {
+              if (!mbar_wait(b.clc, n_resp & 1, wc, 12, kk)) break;
+              ++n_resp;
+              int cx, cy;
+              if (clc_query(clc_resp, cx, cy)) {
+                nx = cx;
+                ny = cy;
+              } else {
+                can_steal = false;
+              }
+            }
+            const int sl = kk & 1;
+            if (!mbar_wait(b.item_empty0 + 8 * sl, ((kk >> 1) & 1) ^ 1, wc, 13, kk)) break;
+            mailbox[2 * sl] = nx;
+            mailbox[2 * sl + 1] = ny;
+            mbar_arrive(b.item_full0 + 8 * sl);   // release: orders the mailbox writes before it
+            if (ny < 0) {
+              k_live = false;
+            } else {
+              ++kk;
+              kj = kseg = koff = 0;
+              prev_h = kh;
+              kq = nx;
+              kh = ny;
+            }
+          } else {
+            next_tile(p, kseg, koff);
+          }
         }
-        if (t >= 1) {
-          const int j = t - 1;
-          const bool chunk = p.seg[vseg].src != 0;
-          const int row = p.seg[vseg].start + voff;
-          const int vs = j % C::VST;
-          if (!mbar_wait(b.v_empty0 + 8 * vs, ((j / C::VST) & 1) ^ 1, wc, 2, j)) break;
-          mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::V_TILE);
-          const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
-          tma_load_4d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0, row, 0, head);
-          nv = j + 1;
-          tr(j, 7);
-          next_tile(p, vseg, voff);
+        if (tv < t - (k_live ? 1 : 0)) {
+          if (!issue_v()) break;
+        } else if (!k_live) {
+          break;
         }
       }
-      // Every load issued must have landed before the CTA may exit.  Older tiles of
-      // a stage completed before the stage was refilled, so the last KST (VST) suffice.
-      mbar_wait_drain(b.q_full, 0, DRAIN_LIMIT_NS);
-      for (int t = nk > C::KST ? nk - C::KST : 0; t < nk; ++t)
-        mbar_wait_drain(b.k_full0 + 8 * (t % C::KST), (t / C::KST) & 1, DRAIN_LIMIT_NS);
-      for (int t = nv > C::VST ? nv - C::VST : 0; t < nv; ++t)
-        mbar_wait_drain(b.v_full0 + 8 * (t % C::VST), (t / C::VST) & 1, DRAIN_LIMIT_NS);
+      // Every load issued must have landed before the CTA may exit.  Older tiles of a stage
+      // completed before the stage was refilled, so the last KST (VST) suffice; likewise the
+      // last Q tile and an unconsumed try_cancel response.
+      if (nq > 0) mbar_wait_drain(b.q_full, (nq - 1) & 1, DRAIN_LIMIT_NS);
+      for (int g = t > C::KST ? t - C::KST : 0; g < t; ++g)
+        mbar_wait_drain(b.k_full0 + 8 * (g % C::KST), (g / C::KST) & 1, DRAIN_LIMIT_NS);
+      for (int g = tv > C::VST ? tv - C::VST : 0; g < tv; ++g)
+        mbar_wait_drain(b.v_full0 + 8 * (g % C::VST), (g / C::VST) & 1, DRAIN_LIMIT_NS);
+      if (n_req > n_resp) mbar_wait_drain(b.clc, n_resp & 1, DRAIN_LIMIT_NS);
     }
     __syncwarp();
   } else if (warp == WARP_MMA) {
@@ -319,13 +418,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       bool ok = mbar_wait(b.q_full, 0, wc, 3, 0);
       tr(0, 14);   // Q tile landed
       tc_fence_after();
-      auto issue_s = [&](int j) -> bool {
-        const int ks = j % C::KST;
-        if (!mbar_wait(b.k_full0 + 8 * ks, (j / C::KST) & 1, wc, 4, j)) return false;
-        if (j > 0) tr(j, 15);   // K_j landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
+      auto issue_s = [&](int g) -> bool {
+        const int ks = g % C::KST;
+        if (!mbar_wait(b.k_full0 + 8 * ks, (g / C::KST) & 1, wc, 4, g)) return false;
+        if (g > 0) tr(g, 15);   // K_g landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
         tc_fence_after();
         const uint32_t sK = sbase + C::OFF_K + ks * C::K_TILE;
-        const uint32_t d = tmem + C::COL_S0 + (j & 1) * BN;
+        const uint32_t d = tmem + C::COL_S0 + (g & 1) * BN;
         if constexpr (QK8) {
 #pragma unroll
           for (int k = 0; k < HD / 32; ++k)   // K = 32 codes per step inside the 128-byte row
@@ -339,8 +438,21 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                     sw128_desc(sK + (k >> 2) * C::KBOX + kin, 16, 1024), C::IDESC_QK, k > 0 ? 1u : 0u);
           }
         }
-        tc_commit(b.s_full0 + 8 * (j & 1));   // also tells the TMA thread that K_j has been read
+        tc_commit(b.s_full0 + 8 * (g & 1));   // also tells the TMA thread that K_g has been read
         return true;
+      };
+      // End of item k: read the next item from the mailbox; if there is one, wait for its Q and
+      // issue its first two S tiles (after this item's last PV in the stream).
+      auto next_item = [&](int k, int g_next, auto&& s_any) -> bool {
+        const int sl = k & 1;
+        if (!mbar_wait(b.item_full0 + 8 * sl, (k >> 1) & 1, wc, 14, k)) return false;
+        const int head = mailbox[2 * sl + 1];
+        mbar_arrive(b.item_empty0 + 8 * sl);
+        if (head < 0) return false;
+        if (!mbar_wait(b.q_full, (k + 1) & 1, wc, 3, k + 1)) return false;
+        tc_fence_after();
+        if (!s_any(g_next)) return false;
+        return n_tiles < 2 || s_any(g_next + 1);
       };
       if constexpr (!QK8 && C::KST == 2 && C::VST == 2) {
         // The production shape.  A UMMA stream issues at the full tensor rate only when the
@@ -361,65 +473,81 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           for (int k = 0; k < BN / 16; ++k)
             dv[h][k] = sw128_desc(sbase + C::OFF_V + h * C::V_TILE + k * 2048, C::KBOX, 1024);
         }
-        auto s_tile = [&](int j, int h) -> bool {   // S_j into buffer h = j & 1 from K stage h
-          if (!mbar_wait(b.k_full0 + 8 * h, (j >> 1) & 1, wc, 4, j)) return false;
-          if (j > 0) tr(j, 15);   // K_j landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
+        auto s_tile = [&](int g, int h) -> bool {   // S_g into buffer h = g & 1 from K stage h
+          if (!mbar_wait(b.k_full0 + 8 * h, (g >> 1) & 1, wc, 4, g)) return false;
+          if (g > 0) tr(g, 15);   // K_g landed (seen by the UMMA thread); tile 0's slot 15 is the CTA's
           tc_fence_after();
           const uint32_t d = tmem + C::COL_S0 + h * BN;
 #pragma unroll
           for (int k = 0; k < HD / 16; ++k) umma_ss(d, dq[k], dk[h][k], C::IDESC_QK, k > 0 ? 1u : 0u);
-          tc_commit(b.s_full0 + 8 * h);   // also tells the TMA thread that K_j has been read
+          tc_commit(b.s_full0 + 8 * h);   // also tells the TMA thread that K_g has been read
           return true;
         };
+        auto s_any = [&](int g) -> bool { return (g & 1) ? s_tile(g, 1) : s_tile(g, 0); };
         if (ok) ok = s_tile(0, 0);
         if (ok && n_tiles > 1) ok = s_tile(1, 1);
-        for (int j0 = 0; ok && j0 < n_tiles; j0 += 2) {
+        for (int k = 0; ok; ++k) {
+          const int base = k * n_tiles, end = base + n_tiles;
+          for (int g0 = base & ~1; ok && g0 < end; g0 += 2) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int j = j0 + h;
-            if (!ok || j >= n_tiles) break;
-            if (!mbar_wait(b.p_full0 + 8 * h, (j >> 1) & 1, wc, 5, j)) {
-              ok = false;
-              break;
-            }
-            tr(j, 3);
-            if (!mbar_wait(b.v_full0 + 8 * h, (j >> 1) & 1, wc, 6, j)) {
-              ok = false;
-              break;
-            }
-            tr(j, 11);
-            tc_fence_after();
-            const uint32_t a = tmem + C::COL_S0 + h * BN;   // P_j, packed bf16, aliases S_j
+            for (int h = 0; h < 2; ++h) {
+              const int g = g0 + h;
+              if (g < base) continue;
+              if (!ok || g >= end) break;
+              if (!mbar_wait(b.p_full0 + 8 * h, (g >> 1) & 1, wc, 5, g)) {
+                ok = false;
+                break;
+              }
+              tr(g, 3);
+              if (!mbar_wait(b.v_full0 + 8 * h, (g >> 1) & 1, wc, 6, g)) {
+                ok = false;
+                break;
+              }
+              tr(g, 11);
+              tc_fence_after();
+              const uint32_t a = tmem + C::COL_S0 + h * BN;   // P_g, packed bf16, aliases S_g
 #pragma unroll
-            for (int k = 0; k < BN / 16; ++k)
-              umma_ts(tmem + C::COL_O, a + 8 * k, dv[h][k], C::IDESC_PV, (j > 0 || k > 0) ? 1u : 0u);
-            tc_commit(b.v_empty0 + 8 * h);   // V_j read, and O holds tiles 0..j
-            tr(j, 4);
-            if (j + 2 < n_tiles) ok = s_tile(j + 2, h);
-            tr(j, 5);
+              for (int kk = 0; kk < BN / 16; ++kk)
+                umma_ts(tmem + C::COL_O, a + 8 * kk, dv[h][kk], C::IDESC_PV, (g > base || kk > 0) ? 1u : 0u);
+              tc_commit(b.v_empty0 + 8 * h);   // V_g read, and O holds the item's tiles up to g
+              tr(g, 4);
+              if (g + 2 < end) ok = s_tile(g + 2, h);
+              tr(g, 5);
+            }
           }
+          if (ok) ok = next_item(k, end, s_any);
         }
       } else {
         if (ok) ok = issue_s(0);
         if (ok && n_tiles > 1) ok = issue_s(1);
-        for (int j = 0; ok && j < n_tiles; ++j) {
-          const int vs = j % C::VST;
-          if (!mbar_wait(b.p_full0 + 8 * (j & 1), (j >> 1) & 1, wc, 5, j)) break;
-          tr(j, 3);
-          if (!mbar_wait(b.v_full0 + 8 * vs, (j / C::VST) & 1, wc, 6, j)) break;
-          tr(j, 11);
-          tc_fence_after();
-          const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
-          const uint32_t a = tmem + C::COL_S0 + (j & 1) * BN;   // P_j, packed bf16, aliases S_j
+        for (int k = 0; ok; ++k) {
+          const int base = k * n_tiles, end = base + n_tiles;
+          for (int g = base; ok && g < end; ++g) {
+            const int vs = g % C::VST;
+            if (!mbar_wait(b.p_full0 + 8 * (g & 1), (g >> 1) & 1, wc, 5, g)) {
+              ok = false;
+              break;
+            }
+            tr(g, 3);
+            if (!mbar_wait(b.v_full0 + 8 * vs, (g / C::VST) & 1, wc, 6, g)) {
+              ok = false;
+              break;
+            }
+            tr(g, 11);
+            tc_fence_after();
+            const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
+            const uint32_t a = tmem + C::COL_S0 + (g & 1) * BN;   // P_g, packed bf16, aliases S_g
 #pragma unroll
-          for (int k = 0; k < BN / 16; ++k) {
-            umma_ts(tmem + C::COL_O, a + 8 * k, sw128_desc(sV + k * 2048, C::KBOX, 1024), C::IDESC_PV,
-                    (j > 0 || k > 0) ? 1u : 0u);
+            for (int kk = 0; kk < BN / 16; ++kk) {
+              umma_ts(tmem + C::COL_O, a + 8 * kk, sw128_desc(sV + kk * 2048, C::KBOX, 1024), C::IDESC_PV,
+                      (g > base || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(b.v_empty0 + 8 * vs);   // V_g read, and O holds the item's tiles up to g
+            tr(g, 4);
+            if (g + 2 < end) ok = issue_s(g + 2);
+            tr(g, 5);
           }
-          tc_commit(b.v_empty0 + 8 * vs);   // V_j read, and O holds tiles 0..j
-          tr(j, 4);
-          if (j + 2 < n_tiles) ok = issue_s(j + 2);
-          tr(j, 5);
+          if (ok) ok = next_item(k, end, issue_s);
         }
       }
       // All UMMAs must have finished before TMEM is released.
@@ -432,18 +560,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int quarter = warp & 3;          // TMEM lane quarter = row block
     const int half = warp >> 2;            // score / output column half
     const int row = quarter * 32 + lane;
-    const int qrow = q0 + row;
-    const bool row_ok = qrow < p.n_q;
     const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int D = p.num_heads * HD;
-    // log2-domain score scale; with 8-bit Q and K it also carries the per-head code scales,
-    // which differ between ring keys and chunk keys
+    int q_tile = blockIdx.x, head = blockIdx.y;   // the current item
+    int qrow = 0;
+    bool row_ok = false;
     float sl2_ring = p.scale_log2, sl2_chunk = p.scale_log2;
-    if constexpr (QK8) {
-      const float qs = p.q_scale[static_cast<int64_t>(head) * gridDim.x + q_tile];   // [H][query blocks]
-      sl2_ring = p.scale_log2 * qs * p.kr_scale[head];
-      sl2_chunk = p.scale_log2 * qs * p.kc_scale[head];
-    }
     float m_run = -INFINITY, l_run = 0.f;  // l_run: this warp's column half only
     int seg = 0, off = 0;
     bool ok = true;
@@ -508,9 +630,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     };
 
     const int pair_id = 2 + quarter;   // named barrier of the warp pair (quarter, quarter + 4)
-    // O holds tiles 0..j once PV_j has completed: the commit that frees V_j's stage.
-    auto wait_o = [&](int j, int site) {
-      return warp_ok(mbar_wait(b.v_empty0 + 8 * (j % C::VST), (j / C::VST) & 1, wc, site, j));
+    // O holds the item's tiles up to g once PV_g has completed: the commit that frees V_g's stage.
+    auto wait_o = [&](int g, int site) {
+      return warp_ok(mbar_wait(b.v_empty0 + 8 * (g % C::VST), (g / C::VST) & 1, wc, site, g));
     };
     // Exchange a value and the status within the warp pair; returns the partner's value and
     // whether both warps are ok.  Two pair barriers: the slots are free again on return.
@@ -561,105 +683,134 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       return fmaxf(fmaxf(fmaxf(m[0], m[1]), fmaxf(m[2], m[3])), fmaxf(fmaxf(m[4], m[5]), fmaxf(m[6], m[7])));
     };
 
-    // Every warp walks every tile and executes the same barriers whether or not it is ok:
-    // the pair barriers of each tile, the snapshot and the epilogue.
-    for (int j = 0; j < n_tiles; ++j) {
-      const int sb = j & 1;
-      if (p.dual && j == p.n_local_tiles && j > 0) {
-        // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
-        if (ok) ok = wait_o(j - 1, 7);
-        if (ok) tc_fence_after();
-        emit(ok, p.out_loc, p.lse_loc, false);
+    // Every warp walks every tile of its items and executes the same barriers whether or not it
+    // is ok: the pair barriers of each tile, the snapshot and the epilogue.
+    for (int k = 0;; ++k) {
+      const int base = k * n_tiles;
+      qrow = q_tile * BM + row;
+      row_ok = qrow < p.n_q;
+      // log2-domain score scale; with 8-bit Q and K it also carries the per-head code scales,
+      // which differ between ring keys and chunk keys
+      if constexpr (QK8) {
+        const int n_qt = (p.n_q + BM - 1) / BM;
+        const float qs = p.q_scale[static_cast<int64_t>(head) * n_qt + q_tile];   // [H][query blocks]
+        sl2_ring = p.scale_log2 * qs * p.kr_scale[head];
+        sl2_chunk = p.scale_log2 * qs * p.kc_scale[head];
       }
-      if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (j >> 1) & 1, wc, 8, j));
-      if (threadIdx.x == 0) tr(j, 0);
-      if (lane == 0) tr(j, 24 + warp);
-      int vloc = min(BN, p.seg[seg].count - off) - half * HALF_COLS;   // valid columns of this half
-      if (p.causal_p != 0 && p.seg[seg].src != 0) {
-        // frame-causal chunk: this row sees chunk keys below the end of its own frame
-        const int kc0 = p.seg[seg].start + off + half * HALF_COLS;   // chunk index of column 0
-        vloc = min(vloc, (qrow / p.causal_p + 1) * p.causal_p - kc0);
-      }
-      const float sl2 = p.seg[seg].src != 0 ? sl2_chunk : sl2_ring;
-      const uint32_t scol = trow + C::COL_S0 + sb * BN + half * HALF_COLS;
-      // load this half's scores (masked columns -inf)
-      auto load_s = [&](uint32_t* s) {
-        tc_fence_after();
-#pragma unroll
-        for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
-#pragma unroll
-        for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
-        if (vloc < HALF_COLS) {
-#pragma unroll
-          for (int i = 0; i < HALF_COLS; ++i)
-            if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
+      m_run = -INFINITY;
+      l_run = 0.f;
+      seg = off = 0;
+      for (int j = 0; j < n_tiles; ++j) {
+        const int g = base + j;
+        const int sb = g & 1;
+        if (p.dual && j == p.n_local_tiles && j > 0) {
+          // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
+          if (ok) ok = wait_o(g - 1, 7);
+          if (ok) tc_fence_after();
+          emit(ok, p.out_loc, p.lse_loc, false);
         }
-      };
-      // P_j overwrites the first 96 columns of S_j (this half's 48 packed columns), so both
-      // halves of the pair must have read their scores first: the pair barrier below orders it.
-      const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
-      uint32_t s[HALF_COLS];
-      float mx = -INFINITY;
-      if (ok) {
-        load_s(s);
-        if (threadIdx.x == 0) tr(j, 8);
-        mx = raw_max(s);
-      }
-      if (threadIdx.x == 0) tr(j, 9);
-      if (j == 0) {
-        // first tile: the row max comes from both halves
-        float mo;
-        ok = pair_exchange(mx, mo);
-        m_run = fmaxf(mx, mo) * sl2;
-      } else {
-        // the running max stands unless the tile's max exceeds it by more than 2^8 somewhere in
-        // the pair's rows (rare); then O is rescaled first
-        const bool need = ok && mx * sl2 > m_run + RESCALE_THRESHOLD;
-        if (pair_or(pair_id, need || !ok)) {
+        if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (g >> 1) & 1, wc, 8, g));
+        if (threadIdx.x == 0) tr(g, 0);
+        if (lane == 0) tr(g, 24 + warp);
+        int vloc = min(BN, p.seg[seg].count - off) - half * HALF_COLS;   // valid columns of this half
+        if (p.causal_p != 0 && p.seg[seg].src != 0) {
+          // frame-causal chunk: this row sees chunk keys below the end of its own frame
+          const int kc0 = p.seg[seg].start + off + half * HALF_COLS;   // chunk index of column 0
+          vloc = min(vloc, (qrow / p.causal_p + 1) * p.causal_p - kc0);
+        }
+        const float sl2 = p.seg[seg].src != 0 ? sl2_chunk : sl2_ring;
+        const uint32_t scol = trow + C::COL_S0 + sb * BN + half * HALF_COLS;
+        // load this half's scores (masked columns -inf)
+        auto load_s = [&](uint32_t* s) {
+          tc_fence_after();
+#pragma unroll
+          for (int i = 0; i < HALF_COLS / 8; ++i) tmem_ld8(scol + 8 * i, s + 8 * i);
+#pragma unroll
+          for (int i = 0; i < HALF_COLS / 8; ++i) tmem_wait_ld8(s + 8 * i);
+          if (vloc < HALF_COLS) {
+#pragma unroll
+            for (int i = 0; i < HALF_COLS; ++i)
+              if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
+          }
+        };
+        // P_j overwrites the first 96 columns of S_j (this half's 48 packed columns), so both
+        // halves of the pair must have read their scores first: the pair barrier below orders it.
+        const uint32_t pcol = trow + C::COL_S0 + sb * BN + half * P_HALF;
+        uint32_t s[HALF_COLS];
+        float mx = -INFINITY;
+        if (ok) {
+          load_s(s);
+          if (threadIdx.x == 0) tr(g, 8);
+          mx = raw_max(s);
+        }
+        if (threadIdx.x == 0) tr(g, 9);
+        if (j == 0) {
+          // first tile: the row max comes from both halves
           float mo;
           ok = pair_exchange(mx, mo);
-          // O holds PV of tiles 0..j-1 once PV_j-1 has completed; lanes whose max did not grow
-          // keep alpha = 1.
-          if (ok) ok = wait_o(j - 1, 9);
-          if (ok) {
-            tc_fence_after();
-            const float m_new = fmaxf(m_run, fmaxf(mx, mo) * sl2);
-            const float alpha = m_new == m_run ? 1.f : ex2_approx(m_run - m_new);
-            l_run *= alpha;
+          m_run = fmaxf(mx, mo) * sl2;
+        } else {
+          // the running max stands unless the tile's max exceeds it by more than 2^8 somewhere in
+          // the pair's rows (rare); then O is rescaled first
+          const bool need = ok && mx * sl2 > m_run + RESCALE_THRESHOLD;
+          if (pair_or(pair_id, need || !ok)) {
+            float mo;
+            ok = pair_exchange(mx, mo);
+            // O holds PV of tiles 0..j-1 once PV_j-1 has completed; lanes whose max did not grow
+            // keep alpha = 1.
+            if (ok) ok = wait_o(g - 1, 9);
+            if (ok) {
+              tc_fence_after();
+              const float m_new = fmaxf(m_run, fmaxf(mx, mo) * sl2);
+              const float alpha = m_new == m_run ? 1.f : ex2_approx(m_run - m_new);
+              l_run *= alpha;
 #pragma unroll 1
-            for (int c = 0; c < C::O_HALF / 8; ++c) {
-              uint32_t r[8];
-              const uint32_t ocol = trow + C::COL_O + half * C::O_HALF + 8 * c;
-              tmem_ld8(ocol, r);
-              tmem_wait_ld8(r);
+              for (int c = 0; c < C::O_HALF / 8; ++c) {
+                uint32_t r[8];
+                const uint32_t ocol = trow + C::COL_O + half * C::O_HALF + 8 * c;
+                tmem_ld8(ocol, r);
+                tmem_wait_ld8(r);
 #pragma unroll
-              for (int i = 0; i < 8; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-              tmem_st4(ocol, r);
-              tmem_st4(ocol + 4, r + 4);
+                for (int i = 0; i < 8; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                tmem_st4(ocol, r);
+                tmem_st4(ocol + 4, r + 4);
+              }
+              tmem_wait_st();
+              m_run = m_new;
             }
-            tmem_wait_st();
-            m_run = m_new;
           }
         }
+        if (threadIdx.x == 0) tr(g, 1);
+        if (ok) {
+          l_run += exps_store(s, sl2, m_run, pcol);
+          if (threadIdx.x == 0) tr(g, 10);
+          tmem_wait_st();
+          tc_fence_before();
+          mbar_arrive(b.p_full0 + 8 * sb);
+          if (threadIdx.x == 0) tr(g, 2);
+          if (lane == 0) tr(g, 16 + warp);
+        }
+        next_tile(p, seg, off);
       }
-      if (threadIdx.x == 0) tr(j, 1);
-      if (ok) {
-        l_run += exps_store(s, sl2, m_run, pcol);
-        if (threadIdx.x == 0) tr(j, 10);
-        tmem_wait_st();
-        tc_fence_before();
-        mbar_arrive(b.p_full0 + 8 * sb);
-        if (threadIdx.x == 0) tr(j, 2);
-        if (lane == 0) tr(j, 16 + warp);
+      {
+        if (ok) ok = wait_o(base + n_tiles - 1, 11);
+        if (ok) tc_fence_after();
+        if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
+        emit(ok, p.out, p.lse, p.dual != 0);
+        if (threadIdx.x == 0 && k == 0) tr(0, 15);   // epilogue stored
       }
-      next_tile(p, seg, off);
-    }
-    {
-      if (ok) ok = wait_o(n_tiles - 1, 11);
-      if (ok) tc_fence_after();
-      if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
-      emit(ok, p.out, p.lse, p.dual != 0);
-      if (threadIdx.x == 0) tr(0, 15);   // epilogue stored
+      // The next item's first PV (which overwrites O) waits for P'_0, which every softmax thread
+      // publishes only after its epilogue's TMEM loads of O have completed.
+      if (!ok) break;
+      const int sl = k & 1;
+      ok = warp_ok(mbar_wait(b.item_full0 + 8 * sl, (k >> 1) & 1, wc, 15, k));
+      if (!ok) break;
+      const int nx = mailbox[2 * sl], ny = mailbox[2 * sl + 1];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b.item_empty0 + 8 * sl);
+      if (ny < 0) break;
+      q_tile = nx;
+      head = ny;
     }
   }
 

@@ -147,6 +147,44 @@ __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, u
   return true;
 }
 
+// ---------------------------------------------------------------- cluster launch control
+// Work stealing between the CTAs of one grid (sm_100 family): try_cancel asks the hardware to
+// cancel one CTA of this grid that has not started yet; the 16-byte response lands in shared
+// memory and completes `bar` as 16 transaction bytes.  A cancelled CTA never runs, so the
+// requesting CTA does its work.  Once a request has failed (nothing left to cancel) no further
+// request may be issued.
+__device__ __forceinline__ void clc_try_cancel(uint32_t resp_smem, uint32_t bar) {
+  asm volatile(
+      "clusterlaunchcontrol.try_cancel.async.shared::cta.mbarrier::complete_tx::bytes.b128 [%0], [%1];" ::"r"(
+          resp_smem),
+      "r"(bar)
+      : "memory");
+}
+// Order this thread's earlier generic-proxy reads of the response buffer before the next
+// try_cancel writes it through the async proxy.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// Decode a completed response: true and the cancelled CTA's (blockIdx.x, blockIdx.y) if a CTA
+// was cancelled, false if the request failed.
+__device__ __forceinline__ bool clc_query(uint32_t resp_smem, int& x, int& y) {
+  uint32_t ok, cx = 0, cy = 0;
+  asm volatile(
+      "{\n\t.reg .b128 rr;\n\t.reg .pred p;\n\t.reg .b64 lo, hi;\n\t"
+      "ld.shared.v2.b64 {lo, hi}, [%3];\n\t"
+      "mov.b128 rr, {lo, hi};\n\t"
+      "clusterlaunchcontrol.query_cancel.is_canceled.pred.b128 p, rr;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t"
+      "@p clusterlaunchcontrol.query_cancel.get_first_ctaid::x.b32.b128 %1, rr;\n\t"
+      "@p clusterlaunchcontrol.query_cancel.get_first_ctaid::y.b32.b128 %2, rr;\n\t}"
+      : "=r"(ok), "+r"(cx), "+r"(cy)
+      : "r"(resp_smem)
+      : "memory");
+  x = static_cast<int>(cx);
+  y = static_cast<int>(cy);
+  return ok != 0;
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* m) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
