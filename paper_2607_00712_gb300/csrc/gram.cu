@@ -371,12 +371,12 @@ constexpr int W_OPER = 4 * W_BOX;       // one operand: 64 tokens x 256 features
 constexpr int W_STAGE = 2 * W_OPER;
 constexpr int W_OFF_BAR = W_ST * W_STAGE;
 constexpr int W_N_BAR = 2 * W_ST + 1 + 2 + 1;   // full/empty stages, acc full, acc empty x2, drain
-constexpr int W_OFF_T = (W_OFF_BAR + W_N_BAR * 8 + 16 + 15) / 16 * 16;   // epilogue staging, 8 warps x 4 KB
+constexpr int W_OFF_T = (W_OFF_BAR + W_N_BAR * 8 + 16 + 1023) / 1024 * 1024;   // epilogue staging, 8 warps x 4 KB
 constexpr int W_SMEM = W_OFF_T + 8 * 32 * 32 * 4;
 constexpr int W_BAND = 8;               // tile columns per band of the blocked order
 constexpr uint32_t W_IDESC = idesc_bf16(128, 256, true, true);
 static_assert(W_SMEM <= 232448, "shared memory per CTA");
-static_assert(W_OFF_T % 16 == 0, "16-byte aligned staging buffers");
+static_assert(W_OFF_T % 1024 == 0, "staging blocks on the 1 KB period of the 128-byte swizzle");
 static_assert(W_STAGE % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
 
 struct WideParams {
@@ -471,7 +471,8 @@ __device__ __forceinline__ bool wit_next(const WideParams& p, WIter& it, WSeg& s
 
 __global__ void __launch_bounds__(W_THREADS, 1)
     gram_wide_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_hi,
-                     const __grid_constant__ CUtensorMap tm_lo, const WideParams p) {
+                     const __grid_constant__ CUtensorMap tm_lo, const __grid_constant__ CUtensorMap tm_state,
+                     const WideParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw;
   const uint32_t sbase = smem_u32(smem);
@@ -581,10 +582,17 @@ __global__ void __launch_bounds__(W_THREADS, 1)
     // ------------------------------------------------------------ epilogue (warps 2-9)
     // warps 2-5 drain the upper accumulator, 6-9 the lower one; warp w reads TMEM lanes
     // 32 (w % 4) .. + 31
+    // Each 32 x 32 block goes TMEM -> registers -> this warp's 4 KB staging block (16-byte
+    // chunk q of row r at chunk q ^ (r & 7), the 128-byte swizzle of the state's tensor map) ->
+    // one bulk tensor reduce-add into the fp32 state, performed by the memory system.  The
+    // accumulator is handed back to the UMMA thread as soon as the warp's last TMEM load has
+    // completed, so the next tile's UMMAs overlap the staging and reduction of the last block.
     const int half = (warp - 2) >> 2;
     const int quarter = warp & 3;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + half * 256;
     const int D = p.D;
+    float4* tbuf = reinterpret_cast<float4*>(smem + W_OFF_T) + (warp - 2) * 32 * 8;
+    const uint32_t tbuf_s = smem_u32(tbuf);
     WIter it;
     wit_init(p, it);
     WSeg sg;
@@ -592,17 +600,34 @@ __global__ void __launch_bounds__(W_THREADS, 1)
     while (wit_next(p, it, sg)) {
       if (!__all_sync(0xffffffffu, mbar_wait(accf, m & 1, wc, 33, m))) break;
       tc_fence_after();
-      const int row0 = (sg.kind == 2 ? D : 0) + sg.bi * 256 + half * 128;
+      const int row0 = (sg.kind == 2 ? D : 0) + sg.bi * 256 + half * 128 + quarter * 32;
       const int col0 = (sg.kind == 0 ? 0 : D) + sg.bj * 256;
-      float4* tbuf = reinterpret_cast<float4*>(smem + W_OFF_T) + (warp - 2) * 32 * 8;
-      float* gblk = p.gram + static_cast<size_t>(row0 + quarter * 32) * (2 * D) + col0;
 #pragma unroll 1
-      for (int c = 0; c < 256 / 32; ++c)
-        flush_block32(lane_base + 32 * c, tbuf, gblk + 32 * c, 2 * static_cast<size_t>(D), lane);
-      tc_fence_before();
-      mbar_arrive(acce0 + 8 * half);
+      for (int c = 0; c < 256 / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(lane_base + 32 * c, v);
+        tmem_wait_ld32(v);
+        if (c == 256 / 32 - 1) {
+          tc_fence_before();
+          mbar_arrive(acce0 + 8 * half);   // accumulator may be overwritten
+        }
+        if (lane == 0) bulk_wait_read_all();   // the previous block's reduce has read the staging block
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          tbuf[lane * 8 + (q ^ (lane & 7))] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                                          __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+        fence_proxy_async_smem();   // these generic-proxy writes before the bulk copy reads them
+        __syncwarp();
+        if (lane == 0) {
+          tma_reduce_add_2d(&tm_state, tbuf_s, col0 + 32 * c, row0);
+          bulk_commit_group();
+        }
+      }
       ++m;
     }
+    if (lane == 0) bulk_wait_all();   // every reduce done before the CTA exits
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -626,11 +651,15 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   }
   // [T][D] operands viewed as (64 features, T tokens, D/64 feature blocks); one box
   // (64, GK, 4) is a 256-feature slice of GK tokens as 4 swizzled [GK][128 B] blocks
-  CUtensorMap tm[3];
+  CUtensorMap tm[3], tm_state;
   const void* srcs[3] = {a_loc, hi, lo};
   for (int i = 0; i < 3; ++i)
     if (!encode_tmap_3d(&tm[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, 4))
       return cudaErrorInvalidValue;
+  // the fp32 [2D][2D] state, 32 x 32 boxes of 128-byte rows
+  if (!encode_tmap_2d_f32(&tm_state, gram, 2 * static_cast<uint64_t>(D), 2 * static_cast<uint64_t>(D),
+                          2 * static_cast<uint64_t>(D) * 4, 32, 32))
+    return cudaErrorInvalidValue;
   WideParams p;
   p.D = D;
   p.NB = D / 256;
@@ -655,7 +684,7 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   p.status = status;
   p.wait_limit_ns = wait_limit_ns;
   p.heartbeat = hb;
-  gram_wide_kernel<<<grid, W_THREADS, W_SMEM, s>>>(tm[0], tm[1], tm[2], p);
+  gram_wide_kernel<<<grid, W_THREADS, W_SMEM, s>>>(tm[0], tm[1], tm[2], tm_state, p);
   return cudaGetLastError();
 }
 

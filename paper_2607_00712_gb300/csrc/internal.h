@@ -133,6 +133,9 @@ bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], c
 bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
                     uint64_t stride1_bytes, uint32_t b0, uint32_t b1);
 // uint8 elements, 128-byte swizzle, rank 2.
+// fp32 [d1][d0] with 128-byte swizzle (the Gram state, for bulk reduce-adds)
+bool encode_tmap_2d_f32(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
+                        uint32_t b0, uint32_t b1);
 bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
                        uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();
