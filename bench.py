@@ -620,6 +620,7 @@ def run_extras(r, wl, device, reps=20):
         dW.zero_()
     out.update(run_w8a8(r, wl, device, W, dW, reps))
     out.update(run_qk8(r, wl, device, reps))
+    out.update(run_kv8(r, wl, device, reps))
     return out
 
 
@@ -672,6 +673,62 @@ def run_qk8(r, wl, device, reps, seed=0):
     tf = wl["flops_full"] / (t_a * 1e-3) / 1e12
     return dict(qk8_full_ms=round(t_a, 4), qk8_full_tflops=round(tf, 1),
                 qk8_chunk_quant_ms=round(t_q, 4), qk8_nk=F * P + nq)
+
+
+def run_kv8(r, wl, device, reps, seed=0):
+    """The F-layer attention with 8-bit Q K^T and 8-bit P V (e4m3 keys and d-major e4m3 values in
+    the ring, e4m3 probabilities in the kernel) on the same history as the step's F-layer ring;
+    per step the chunk's queries, keys and values are quantised (timed separately).  L2 is
+    flushed before every repetition."""
+    import torch
+    from paper_2607_00712_gb300 import synth
+    from paper_2607_00712_gb300.device import Ring, bf16_tensor
+    abi = r.abi
+    H, d, P, L, F, nq = (wl[k] for k in ("H", "d", "P", "L", "F", "nq"))
+    if d != 128 or P % 4:
+        return {}
+    s = synth.make_step(seed * 100 + 0, F, P, H, d, L)          # the F-layer ring's inputs
+    kh = bf16_tensor(s.k_hist, device)
+    vh = bf16_tensor(s.v_hist, device)
+    n_hist = kh.shape[0]
+    scratch = torch.empty(n_hist, H, d, dtype=torch.uint8, device=device)
+    k_scale = torch.empty(H, dtype=torch.float32, device=device)
+    v_scale = torch.empty(H, dtype=torch.float32, device=device)
+    abi.ispa_quantize_heads_e4m3(kh, n_hist, H, d, scratch, k_scale)
+    abi.ispa_quantize_heads_e4m3(vh, n_hist, H, d, scratch, v_scale)
+    ring = Ring(H, d, P, F, 0, device, kv_e4m3=True)
+    for f0 in range(0, F, L):
+        n = min(L, F - f0)
+        abi.ispa_kv_append_kv8(ring.c, kh[f0 * P:(f0 + n) * P], vh[f0 * P:(f0 + n) * P], n, k_scale, v_scale)
+    del scratch, kh, vh
+    q, kc, vc = r.inputs[0]
+    q8 = torch.empty(nq, H, d, dtype=torch.uint8, device=device)
+    k8 = torch.empty_like(q8)
+    qs = torch.empty(H, (nq + 127) // 128, dtype=torch.float32, device=device)
+    ld = (nq + 15) // 16 * 16
+    vt8 = torch.empty(H, d, ld, dtype=torch.uint8, device=device)
+    out = torch.empty(nq, H * d, dtype=torch.bfloat16, device=device)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=device)
+    st = r.stream
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    t_q = t_a = 0.0
+    for i in range(reps + 3):
+        flush.fill_(float(i))
+        ev[0].record(st)
+        abi.ispa_quantize_q_e4m3(q, nq, H, d, q8, qs, st)
+        abi.ispa_quantize_k_e4m3(kc, nq, H, d, k_scale, k8, st)
+        abi.ispa_quantize_vt_e4m3(vc, nq, H, d, v_scale, vt8, ld, st)
+        ev[1].record(st)
+        abi.ispa_attn_full_kv8(ring.c, k_scale, v_scale, q8, qs, k8, k_scale, vt8, ld, nq, 0.0, out, None, st)
+        ev[2].record(st)
+        torch.cuda.synchronize(device)
+        if i >= 3:
+            t_q += ev[0].elapsed_time(ev[1])
+            t_a += ev[1].elapsed_time(ev[2])
+    t_q, t_a = t_q / reps, t_a / reps
+    tf = wl["flops_full"] / (t_a * 1e-3) / 1e12
+    return dict(kv8_full_ms=round(t_a, 4), kv8_full_tflops=round(tf, 1), kv8_chunk_quant_ms=round(t_q, 4),
+                kv8_ring_bytes=int(abi.ispa_ring_bytes(ring.c)))
 
 
 def run_w8a8(r, wl, device, W, dW, reps):

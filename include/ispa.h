@@ -89,12 +89,17 @@ typedef enum {
  *   buffers) checkpoints the cache.  With k_format = ISPA_KV_K_E4M3, k holds
  *   e4m3 codes [H][capacity_frames * P][head_dim] (one byte each; head_dim 128)
  *   written by ispa_kv_append_qk8 with one fp32 scale per head that the caller
- *   keeps for the ring's life.  Slots never written must still hold
+ *   keeps for the ring's life.  With k_format = ISPA_KV_KV_E4M3 (head_dim 128,
+ *   P % 4 == 0), k holds those key codes and v holds the values as e4m3 codes
+ *   d-major, [H][head_dim][ispa_ring_vt_stride(ring)] (key index slot * P + t
+ *   within a row), written by ispa_kv_append_kv8 with the caller's per-head key
+ *   and value scales.  Slots never written must still hold
  *   finite values (zero-fill the buffers at creation): a key tile that ends
  *   inside a run reads the rows after it with weight zero, and 0 * NaN is NaN.
  */
 #define ISPA_KV_BF16 0     /* k_format: keys bf16 (every entry point except *_qk8) */
 #define ISPA_KV_K_E4M3 1   /* k_format: keys e4m3 codes, 1 byte each (the *_qk8 entry points) */
+#define ISPA_KV_KV_E4M3 2  /* k_format: keys and d-major values as e4m3 codes (the *_kv8 entry points) */
 
 typedef struct {
   int32_t num_heads;
@@ -102,7 +107,7 @@ typedef struct {
   int32_t tokens_per_frame;
   int32_t capacity_frames;
   int32_t n_sink_frames;
-  int32_t k_format;       /* ISPA_KV_BF16 or ISPA_KV_K_E4M3; values stay bf16 */
+  int32_t k_format;       /* ISPA_KV_BF16, ISPA_KV_K_E4M3 (values bf16) or ISPA_KV_KV_E4M3 */
   int64_t frames_written;
   void* k;
   void* v;
@@ -543,6 +548,64 @@ ISPA_API ispa_status ispa_attn_dual_qk8(const ispa_kv_ring* ring, const float* k
                                         const void* q8, const float* q_scale, const void* k8_cur,
                                         const float* k_cur_scale, const void* v_cur, int32_t n_q, float scale,
                                         void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
+                                        float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
+                                        ispa_stream stream);
+
+/* ------------------------------------------------------------ 8-bit Q K^T and P V attention */
+/*
+ * SageAttention's second form, which the paper cites for its attention kernels
+ * (Sec. 3.4): Q K^T as above and P V in fp8 too -- the values as e4m3 codes with
+ * one fp32 scale per head, the probabilities rounded to e4m3 in the kernel.  V is
+ * stored d-major ([H][128][keys]), the operand layout of the 8-bit P V.  The result
+ * approximates the attention of the dequantised q, k and v; the difference comes
+ * from the e4m3 rounding of P only.  P_i = 2^(s_i - m) against a running maximum m
+ * that stays within 2^4 of the row's maximum score, scaled by 2^4 before rounding:
+ * each weight p_i = P_i / l (l = sum_i P_i >= 1, exact in fp32) is used with relative
+ * error <= 2^-4, or absolute error <= 2^-14 / l where e4m3 is subnormal, so an
+ * output element differs by at most 2^-4 sum_i p_i |v_i| + 2^-14 sum_i |v_i| / L,
+ * L = sum_i exp(s_i - max_j s_j) <= l, plus the bf16 path's own rounding.  Head dim
+ * 128; tokens per frame a multiple of 4.
+ */
+
+/* Row stride in bytes of a ISPA_KV_KV_E4M3 ring's d-major value codes:
+ * capacity_frames * P rounded up to a multiple of 16. */
+ISPA_API int64_t ispa_ring_vt_stride(const ispa_kv_ring* ring);
+
+/* Values as d-major codes with given per-head scales: x bf16 [n][H][d] (d = 128),
+ * scale fp32 [H] (device) -> qt uint8 [H][d][ld] with qt[h][c][t] =
+ * e4m3(x[t][h][c] * (1 / scale_h)) as in ispa_quantize_k_e4m3; entries t >= n of a
+ * row are left as they are.  ld >= n, ld % 16 == 0.  For the chunk's values,
+ * with the ring's value scales. */
+ISPA_API ispa_status ispa_quantize_vt_e4m3(const void* x, int64_t n, int32_t H, int32_t d, const float* scale,
+                                           uint8_t* qt, int64_t ld, ispa_stream stream);
+
+/* ispa_kv_append for a ring with k_format = ISPA_KV_KV_E4M3: keys coded with the
+ * ring's key scales k_scale[H] as ispa_kv_append_qk8 does, values coded with the
+ * ring's value scales v_scale[H] (device fp32, fixed for the ring's life, e.g. from
+ * ispa_quantize_heads_e4m3 of the first values) into their d-major slots. */
+ISPA_API ispa_status ispa_kv_append_kv8(ispa_kv_ring* ring, const void* k_new, const void* v_new,
+                                        int32_t n_frames, const float* k_scale, const float* v_scale,
+                                        ispa_stream stream);
+
+/* ispa_attn_full_qk8 / ispa_attn_local_qk8 / ispa_attn_dual_qk8 with 8-bit P V over a
+ * ISPA_KV_KV_E4M3 ring:
+ *   v_scale : the ring's value scales (as given to ispa_kv_append_kv8), device fp32 [H]
+ *   vt8_cur : the chunk's values as d-major codes [H][128][vt_ld] with v_scale (from
+ *             ispa_quantize_vt_e4m3), vt_ld >= n_q, vt_ld % 16 == 0
+ * Other arguments and errors as the *_qk8 calls; any other ring is
+ * ISPA_ERR_INVALID_ARG. */
+ISPA_API ispa_status ispa_attn_full_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                                        const void* q8, const float* q_scale, const void* k8_cur,
+                                        const float* k_cur_scale, const void* vt8_cur, int64_t vt_ld, int32_t n_q,
+                                        float scale, void* out, float* lse, ispa_stream stream);
+ISPA_API ispa_status ispa_attn_local_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                                         ispa_window win, const void* q8, const float* q_scale, const void* k8_cur,
+                                         const float* k_cur_scale, const void* vt8_cur, int64_t vt_ld, int32_t n_q,
+                                         float scale, void* out, float* lse, ispa_stream stream);
+ISPA_API ispa_status ispa_attn_dual_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                                        ispa_window win, const void* q8, const float* q_scale, const void* k8_cur,
+                                        const float* k_cur_scale, const void* vt8_cur, int64_t vt_ld, int32_t n_q,
+                                        float scale, void* a_full, void* a_loc, float* disc, float* disc_sq_sum,
                                         float* lse_full, float* lse_loc, void* workspace, size_t ws_bytes,
                                         ispa_stream stream);
 

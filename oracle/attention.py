@@ -60,6 +60,17 @@ def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float):
     return o, lse
 
 
+def attend_weights(q: np.ndarray, k: np.ndarray, scale: float):
+    """The softmax weights of one head, as `attend` forms them: q [n, d], k [m, d] ->
+    (p [n, m], L [n]) with p = exp(s - max s) / L and L = sum exp(s - max s), s = scale q k^T."""
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    s = scale * (q @ k.T)
+    e = np.exp(s - s.max(axis=1)[:, None])
+    L = e.sum(axis=1)
+    return e / L[:, None], L
+
+
 def attend_heads(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float):
     """All heads: q [n, H, d], k/v [m, H, d] -> (o [n, H, d], lse [H, n])."""
     n, H, _ = q.shape

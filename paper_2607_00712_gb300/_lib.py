@@ -27,6 +27,7 @@ ISPA_ERR_WORKSPACE = 7
 ISPA_ATTN_FRAME_CAUSAL = 1   # option bit of the *_ex attention entry points
 ISPA_KV_BF16 = 0             # ring k_format values
 ISPA_KV_K_E4M3 = 1
+ISPA_KV_KV_E4M3 = 2
 MAX_RANGES = 4
 
 
@@ -119,6 +120,16 @@ _SIGS = {
     "ispa_quantize_q_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_quantize_k_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_kv_append_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
+    "ispa_ring_vt_stride": (c_int64, [POINTER(KVRing)]),
+    "ispa_quantize_vt_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_int64, c_void_p]),
+    "ispa_kv_append_kv8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_full_kv8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_int64, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_local_kv8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, Window, c_void_p, c_void_p, c_void_p,
+                                      c_void_p, c_void_p, c_int64, c_int32, c_float, c_void_p, c_void_p, c_void_p]),
+    "ispa_attn_dual_kv8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, Window, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_void_p, c_int64, c_int32, c_float, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "ispa_attn_full_qk8": (c_int32, [POINTER(KVRing), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                      c_int32, c_float, c_void_p, c_void_p, c_void_p]),
     "ispa_attn_dual_qk8": (c_int32, [POINTER(KVRing), c_void_p, Window, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -411,6 +422,43 @@ def ispa_quantize_q_e4m3(x, n: int, H: int, d: int, q, scale, stream=None) -> No
 def ispa_quantize_k_e4m3(x, n: int, H: int, d: int, scale, q, stream=None) -> None:
     _check(lib().ispa_quantize_k_e4m3(_ptr(x), n, H, d, _ptr(scale), _ptr(q), _stream(stream)),
            "ispa_quantize_k_e4m3")
+
+
+def ispa_ring_vt_stride(ring: KVRing) -> int:
+    return lib().ispa_ring_vt_stride(ctypes.byref(ring))
+
+
+def ispa_quantize_vt_e4m3(x, n: int, H: int, d: int, scale, qt, ld: int, stream=None) -> None:
+    _check(lib().ispa_quantize_vt_e4m3(_ptr(x), n, H, d, _ptr(scale), _ptr(qt), ld, _stream(stream)),
+           "ispa_quantize_vt_e4m3")
+
+
+def ispa_kv_append_kv8(ring: KVRing, k_new, v_new, n_frames: int, k_scale, v_scale, stream=None) -> None:
+    _check(lib().ispa_kv_append_kv8(ctypes.byref(ring), _ptr(k_new), _ptr(v_new), n_frames, _ptr(k_scale),
+                                    _ptr(v_scale), _stream(stream)), "ispa_kv_append_kv8")
+
+
+def ispa_attn_full_kv8(ring: KVRing, k_ring_scale, v_scale, q8, q_scale, k8_cur, k_cur_scale, vt8_cur, vt_ld: int,
+                       n_q: int, scale: float, out, lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_full_kv8(ctypes.byref(ring), _ptr(k_ring_scale), _ptr(v_scale), _ptr(q8), _ptr(q_scale),
+                                    _ptr(k8_cur), _ptr(k_cur_scale), _ptr(vt8_cur), vt_ld, n_q, scale, _ptr(out),
+                                    _ptr(lse), _stream(stream)), "ispa_attn_full_kv8")
+
+
+def ispa_attn_local_kv8(ring: KVRing, k_ring_scale, v_scale, win: Window, q8, q_scale, k8_cur, k_cur_scale, vt8_cur,
+                        vt_ld: int, n_q: int, scale: float, out, lse=None, stream=None) -> None:
+    _check(lib().ispa_attn_local_kv8(ctypes.byref(ring), _ptr(k_ring_scale), _ptr(v_scale), win, _ptr(q8),
+                                     _ptr(q_scale), _ptr(k8_cur), _ptr(k_cur_scale), _ptr(vt8_cur), vt_ld, n_q, scale,
+                                     _ptr(out), _ptr(lse), _stream(stream)), "ispa_attn_local_kv8")
+
+
+def ispa_attn_dual_kv8(ring: KVRing, k_ring_scale, v_scale, win: Window, q8, q_scale, k8_cur, k_cur_scale, vt8_cur,
+                       vt_ld: int, n_q: int, scale: float, a_full, a_loc, disc, disc_sq_sum, lse_full=None,
+                       lse_loc=None, workspace=None, ws_bytes: int = 0, stream=None) -> None:
+    _check(lib().ispa_attn_dual_kv8(ctypes.byref(ring), _ptr(k_ring_scale), _ptr(v_scale), win, _ptr(q8),
+                                    _ptr(q_scale), _ptr(k8_cur), _ptr(k_cur_scale), _ptr(vt8_cur), vt_ld, n_q, scale,
+                                    _ptr(a_full), _ptr(a_loc), _ptr(disc), _ptr(disc_sq_sum), _ptr(lse_full),
+                                    _ptr(lse_loc), _ptr(workspace), ws_bytes, _stream(stream)), "ispa_attn_dual_kv8")
 
 
 def ispa_attn_dual_qk8(ring: KVRing, k_ring_scale, win: Window, q8, q_scale, k8_cur, k_cur_scale, v_cur, n_q: int,

@@ -196,6 +196,20 @@ bool encode_tmap_4d(CUtensorMap* m, const void* base, const uint64_t dims4[4], c
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_tmap_3d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                       uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1, uint32_t b2) {
+  ensure_context();
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
                        uint32_t b0, uint32_t b1) {
   ensure_context();
@@ -247,8 +261,10 @@ ispa_status check_ring(const ispa_kv_ring* r) {
       r->n_sink_frames < 0 || r->n_sink_frames >= r->capacity_frames || r->frames_written < 0)
     return ISPA_ERR_INVALID_ARG;
   if (r->head_dim != 64 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
-  if (r->k_format != ISPA_KV_BF16 && r->k_format != ISPA_KV_K_E4M3) return ISPA_ERR_INVALID_ARG;
-  if (r->k_format == ISPA_KV_K_E4M3 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
+  if (r->k_format != ISPA_KV_BF16 && r->k_format != ISPA_KV_K_E4M3 && r->k_format != ISPA_KV_KV_E4M3)
+    return ISPA_ERR_INVALID_ARG;
+  if (r->k_format != ISPA_KV_BF16 && r->head_dim != 128) return ISPA_ERR_UNSUPPORTED;
+  if (r->k_format == ISPA_KV_KV_E4M3 && r->tokens_per_frame % 4 != 0) return ISPA_ERR_UNSUPPORTED;
   if (static_cast<int64_t>(r->capacity_frames) * r->tokens_per_frame > INT32_MAX)
     return ISPA_ERR_INVALID_ARG;
   return ISPA_OK;
@@ -327,11 +343,14 @@ int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P, int
   return tiles;
 }
 
-// 8-bit Q K^T: per-head e4m3 code scales of q, of the chunk keys and of the ring keys.
+// 8-bit Q K^T: per-head e4m3 code scales of q, of the chunk keys and of the ring keys; with 8-bit
+// P V also the values' per-head scale and the row stride of the chunk's d-major value codes.
 struct Qk8Scales {
   const float* q;
   const float* k_cur;
   const float* k_ring;
+  const float* v = nullptr;
+  int64_t vt_ld = 0;
 };
 
 ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, const void* q,
@@ -340,8 +359,11 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
                         cudaStream_t stream, const Qk8Scales* qk8 = nullptr) {
   ispa_status st = check_ring(ring);
   if (st != ISPA_OK) return st;
-  if ((ring->k_format == ISPA_KV_K_E4M3) != (qk8 != nullptr)) return ISPA_ERR_INVALID_ARG;
+  if ((ring->k_format != ISPA_KV_BF16) != (qk8 != nullptr)) return ISPA_ERR_INVALID_ARG;
   if (qk8 && (!qk8->q || !qk8->k_cur || !qk8->k_ring)) return ISPA_ERR_INVALID_ARG;
+  const bool kv8 = ring->k_format == ISPA_KV_KV_E4M3;
+  if (kv8 && (!qk8->v || qk8->vt_ld < n_q || qk8->vt_ld % 16 != 0)) return ISPA_ERR_INVALID_ARG;
+  if (!kv8 && qk8 && qk8->v) return ISPA_ERR_INVALID_ARG;   // 8-bit P V needs a ring with e4m3 values
   if (flags & ~static_cast<uint32_t>(ISPA_ATTN_FRAME_CAUSAL)) return ISPA_ERR_INVALID_ARG;
   if ((flags & ISPA_ATTN_FRAME_CAUSAL) && n_q % ring->tokens_per_frame != 0) return ISPA_ERR_INVALID_ARG;
   if (n_q <= 0 || !aligned16(q) || !aligned16(k_cur) || !aligned16(v_cur) || !aligned16(out) ||
@@ -417,7 +439,19 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const uint32_t box_q[4] = {64, static_cast<uint32_t>(kAttnBM), nb, 1};
   const uint32_t box_k[4] = {64, static_cast<uint32_t>(bn), nb, 1};
   CUtensorMap tq, tkr, tvr, tkc, tvc;
-  bool ok = encode_tmap_4d(&tvc, v_cur, dims_c, str_c, box_k) && encode_tmap_4d(&tvr, ring->v, dims_r, str_r, box_k);
+  bool ok;
+  if (kv8) {
+    // d-major e4m3 values [H][128][keys]: boxes of 128 keys x 128 rows, 128-byte swizzle (the
+    // K-major B operand of the 8-bit P V)
+    const uint64_t vt_ring = ispa_ring_vt_stride(ring);
+    ok = encode_tmap_3d_u8(&tvc, v_cur, static_cast<uint64_t>(n_q), 128, static_cast<uint64_t>(H),
+                           static_cast<uint64_t>(qk8->vt_ld), static_cast<uint64_t>(qk8->vt_ld) * 128, 128, 128, 1) &&
+         encode_tmap_3d_u8(&tvr, ring->v, ring_tok, 128, static_cast<uint64_t>(H), vt_ring, vt_ring * 128, 128, 128,
+                           1);
+    p.v_scale = qk8->v;
+  } else {
+    ok = encode_tmap_4d(&tvc, v_cur, dims_c, str_c, box_k) && encode_tmap_4d(&tvr, ring->v, dims_r, str_r, box_k);
+  }
   if (qk8) {
     // e4m3 Q and K: a token's 128 features are one 128-byte row, so the column-block
     // dimension has extent 1
@@ -531,7 +565,15 @@ size_t ispa_ring_bytes(const ispa_kv_ring* r) {
   if (!r || r->num_heads <= 0 || r->head_dim <= 0 || r->tokens_per_frame <= 0 || r->capacity_frames <= 0)
     return 0;
   const uint64_t elems = 1ull * r->num_heads * r->capacity_frames * r->tokens_per_frame * r->head_dim;
+  if (r->k_format == ISPA_KV_KV_E4M3)
+    return elems + 1ull * r->num_heads * r->head_dim * static_cast<uint64_t>(ispa_ring_vt_stride(r));
   return elems * (r->k_format == ISPA_KV_K_E4M3 ? 1ull : 2ull) + elems * 2ull;
+}
+
+int64_t ispa_ring_vt_stride(const ispa_kv_ring* r) {
+  if (!r || r->tokens_per_frame <= 0 || r->capacity_frames <= 0) return 0;
+  const int64_t keys = static_cast<int64_t>(r->capacity_frames) * r->tokens_per_frame;
+  return (keys + 15) / 16 * 16;
 }
 
 int32_t ispa_ring_slot(const ispa_kv_ring* r, int64_t frame) {
@@ -788,6 +830,75 @@ ispa_status ispa_kv_append_qk8(ispa_kv_ring* ring, const void* k_new, const void
                         v_new, ring->k, ring->v, k_scale, stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   ring->frames_written += n_frames;
+  return ISPA_OK;
+}
+
+ispa_status ispa_quantize_vt_e4m3(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* qt,
+                                  int64_t ld, ispa_stream stream) {
+  if (!x || !scale || !qt || n <= 0 || H <= 0 || !aligned16(x) || !aligned16(qt) || ld < n || ld % 16 != 0)
+    return ISPA_ERR_INVALID_ARG;
+  if (d != 128) return ISPA_ERR_UNSUPPORTED;
+  if (launch_quant_vt(x, n, H, d, scale, qt, ld, 0, 0, nullptr, stream) != cudaSuccess) return ISPA_ERR_CUDA;
+  return ISPA_OK;
+}
+
+ispa_status ispa_kv_append_kv8(ispa_kv_ring* ring, const void* k_new, const void* v_new, int32_t n_frames,
+                               const float* k_scale, const float* v_scale, ispa_stream stream) {
+  const ispa_status st = check_ring(ring);
+  if (st != ISPA_OK) return st;
+  if (ring->k_format != ISPA_KV_KV_E4M3 || !k_new || !v_new || !k_scale || !v_scale || n_frames <= 0)
+    return ISPA_ERR_INVALID_ARG;
+  if (!aligned16(ring->k) || !aligned16(ring->v) || !aligned16(k_new) || !aligned16(v_new))
+    return ISPA_ERR_INVALID_ARG;
+  if (n_frames > kMaxAppendFrames || n_frames > ring->capacity_frames - ring->n_sink_frames) return ISPA_ERR_CAPACITY;
+  int32_t slots[kMaxAppendFrames];
+  for (int i = 0; i < n_frames; ++i) slots[i] = slot_of(ring, ring->frames_written + i);
+  const int32_t P = ring->tokens_per_frame;
+  const int64_t ring_tok = static_cast<int64_t>(ring->capacity_frames) * P;
+  if (launch_append_qk8(slots, n_frames, P, ring->num_heads, ring->head_dim, ring_tok, k_new, v_new, ring->k,
+                        nullptr, k_scale, stream) != cudaSuccess ||
+      launch_quant_vt(v_new, static_cast<int64_t>(n_frames) * P, ring->num_heads, ring->head_dim, v_scale,
+                      static_cast<uint8_t*>(ring->v), ispa_ring_vt_stride(ring), P, n_frames, slots,
+                      stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
+  ring->frames_written += n_frames;
+  return ISPA_OK;
+}
+
+ispa_status ispa_attn_full_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                               const void* q8, const float* q_scale, const void* k8_cur, const float* k_cur_scale,
+                               const void* vt8_cur, int64_t vt_ld, int32_t n_q, float scale, void* out, float* lse,
+                               ispa_stream stream) {
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale, v_scale, vt_ld};
+  return attn_common(MODE_FULL, ring, ispa_window{0, 0}, q8, k8_cur, vt8_cur, n_q, scale, 0u, out, nullptr, lse,
+                     nullptr, nullptr, stream, &sc);
+}
+
+ispa_status ispa_attn_local_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                                ispa_window win, const void* q8, const float* q_scale, const void* k8_cur,
+                                const float* k_cur_scale, const void* vt8_cur, int64_t vt_ld, int32_t n_q, float scale,
+                                void* out, float* lse, ispa_stream stream) {
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale, v_scale, vt_ld};
+  return attn_common(MODE_LOCAL, ring, win, q8, k8_cur, vt8_cur, n_q, scale, 0u, out, nullptr, lse, nullptr,
+                     nullptr, stream, &sc);
+}
+
+ispa_status ispa_attn_dual_kv8(const ispa_kv_ring* ring, const float* k_ring_scale, const float* v_scale,
+                               ispa_window win, const void* q8, const float* q_scale, const void* k8_cur,
+                               const float* k_cur_scale, const void* vt8_cur, int64_t vt_ld, int32_t n_q, float scale,
+                               void* a_full, void* a_loc, float* disc, float* disc_sq_sum, float* lse_full,
+                               float* lse_loc, void* workspace, size_t ws_bytes, ispa_stream stream) {
+  if (!ring || !disc || !disc_sq_sum) return ISPA_ERR_INVALID_ARG;
+  const size_t need = ispa_attn_dual_workspace_size(ring->num_heads, n_q);
+  if (need == 0) return ISPA_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
+  float* part = static_cast<float*>(workspace);
+  const Qk8Scales sc{q_scale, k_cur_scale, k_ring_scale, v_scale, vt_ld};
+  const ispa_status st = attn_common(MODE_DUAL, ring, win, q8, k8_cur, vt8_cur, n_q, scale, 0u, a_full, a_loc,
+                                     lse_full, lse_loc, part, stream, &sc);
+  if (st != ISPA_OK) return st;
+  if (launch_disc_reduce(part, ring->num_heads, n_q, disc, disc_sq_sum, stream) != cudaSuccess)
+    return ISPA_ERR_CUDA;
   return ISPA_OK;
 }
 

@@ -71,17 +71,30 @@ constexpr int HALF_COLS = BN / 2;          // score columns per softmax warp
 constexpr int P_HALF = HALF_COLS / 2;      // packed bf16 P columns per softmax warp
 static_assert(BN % 16 == 0 && BN <= 256 && HALF_COLS % 8 == 0 && P_HALF % 4 == 0, "key tile shape");
 
+// PV8 (with QK8): V as e4m3 codes too, from d-major ("transposed") tiles [128 d rows][keys]: the
+// K-major B operand of a kind::f8f6f4 P V with P as e4m3 in TMEM.  A TMA box must start on a
+// 16-byte boundary, so a tile's V window starts at its first key rounded down to a multiple of
+// 16 and covers 256 keys (two 128-key boxes with 128-byte swizzle); P is written into TMEM
+// shifted by the remainder r, with zeros around it, and P V runs as 7 UMMAs of K = 32 over the
+// first 224 keys of the window (r + 192 <= 204).  P is scaled by 2^4 before its e4m3 rounding
+// (the running max is kept within 2^4 of every tile's max, so P' <= 2^8 < 448), which keeps
+// values down to 2^-10 of the row maximum in e4m3's normal range.
 // QK8: Q and K as e4m3 codes (one 128-byte swizzled row = the 128 features of a token), S by
 // kind::f8f6f4 UMMAs with K = 32; V, P and O as in the bf16 path.
-template <int HD, bool QK8 = false>
+template <int HD, bool QK8 = false, bool PV8 = false>
 struct Cfg {
   static_assert(!QK8 || HD == 128, "8-bit Q K^T is built for head_dim 128");
+  static_assert(!PV8 || QK8, "8-bit P V comes with 8-bit Q K^T");
   static constexpr int NBOX = HD / 64;          // 64-column (128-byte) TMA boxes per bf16 tile row
   static constexpr int QBOX = BM * 128;         // [128 rows][64 bf16] = 16 KB
   static constexpr int KBOX = BN * 128;         // [192 rows][64 bf16] = 24 KB
   static constexpr int Q_TILE = QK8 ? BM * HD : NBOX * QBOX;
   static constexpr int K_TILE = QK8 ? BN * HD : NBOX * KBOX;
-  static constexpr int V_TILE = NBOX * KBOX;
+  static constexpr int V_BOX8 = 128 * HD;                  // [HD rows][128 keys] e4m3 = 16 KB
+  static constexpr int V_TILE = PV8 ? 2 * V_BOX8 : NBOX * KBOX;
+  static constexpr int PV_STEPS = PV8 ? 7 : BN / 16;       // UMMAs of one P V
+  static constexpr float RESCALE = PV8 ? 4.0f : RESCALE_THRESHOLD;   // lazy rescale bound (log2)
+  static constexpr float P_SHIFT = PV8 ? 4.0f : 0.0f;      // log2 of the scale P gets before rounding
   static constexpr int KST = (HD == 128 && !QK8) ? 2 : 4;  // K stages
   static constexpr int VST = HD == 128 ? 2 : 4;            // V stages
   static constexpr int OFF_Q = 0;
@@ -102,7 +115,7 @@ struct Cfg {
   static constexpr uint32_t COL_S0 = 0, COL_O = 2 * BN;
   static constexpr int O_HALF = HD / 2;             // O columns per softmax warp
   static constexpr uint32_t IDESC_QK = QK8 ? idesc_e4m3(BM, BN) : idesc_bf16(BM, BN, false, false);
-  static constexpr uint32_t IDESC_PV = idesc_bf16(BM, HD, false, true);
+  static constexpr uint32_t IDESC_PV = PV8 ? idesc_e4m3(BM, HD) : idesc_bf16(BM, HD, false, true);
   static_assert(COL_O + HD <= 512, "TMEM columns");
   static_assert(KBOX % 1024 == 0 && QBOX % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
 };
@@ -196,12 +209,12 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 // epilogue's reads of O.
 // The TMA thread asks for the next item a few tiles before the end of the current one and
 // publishes it (or "none") to the UMMA thread and the softmax warps through a two-slot mailbox.
-template <int HD, bool QK8, bool TRACE>
+template <int HD, bool QK8, bool PV8, bool TRACE>
 __global__ void __launch_bounds__(NTHREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kr,
                 const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_kc,
                 const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
-  using C = Cfg<HD, QK8>;
+  using C = Cfg<HD, QK8, PV8>;
   // The dynamic shared window must start on a 1 KB boundary (the swizzle atoms of the
   // TMA boxes); the declaration asks for it and the check below enforces it.
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -328,8 +341,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (!mbar_wait(b.v_empty0 + 8 * vs, ((tv / C::VST) & 1) ^ 1, wc, 2, tv)) return false;
         const bool chunk = p.seg[vseg].src != 0;
         mbar_arrive_expect_tx(b.v_full0 + 8 * vs, C::V_TILE);
-        tma_load_4d(sbase + C::OFF_V + vs * C::V_TILE, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0,
-                    p.seg[vseg].start + voff, 0, vk == kk ? kh : prev_h);
+        const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
+        const int vhead = vk == kk ? kh : prev_h;
+        if constexpr (PV8) {
+          // d-major e4m3 V: the 256-key window from the tile's first key rounded down to 16
+          const int x0 = (p.seg[vseg].start + voff) & ~15;
+          tma_load_3d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, x0, 0, vhead);
+          tma_load_3d(sV + C::V_BOX8, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, x0 + 128, 0, vhead);
+        } else {
+          tma_load_4d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, 0, p.seg[vseg].start + voff, 0, vhead);
+        }
         tr(tv, 7);
         ++tv;
         if (++vj == n_tiles) {
@@ -536,11 +557,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             tr(g, 11);
             tc_fence_after();
             const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
-            const uint32_t a = tmem + C::COL_S0 + (g & 1) * BN;   // P_g, packed bf16, aliases S_g
+            const uint32_t a = tmem + C::COL_S0 + (g & 1) * BN;   // P_g, packed bf16 or e4m3, aliases S_g
+            if constexpr (PV8) {
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk) {
-              umma_ts(tmem + C::COL_O, a + 8 * kk, sw128_desc(sV + kk * 2048, C::KBOX, 1024), C::IDESC_PV,
-                      (g > base || kk > 0) ? 1u : 0u);
+              for (int kk = 0; kk < C::PV_STEPS; ++kk)   // K = 32 keys (8 TMEM columns, 32 bytes of a V row)
+                umma_f8_ts(tmem + C::COL_O, a + 8 * kk,
+                           sw128_desc(sV + (kk >> 2) * C::V_BOX8 + (kk & 3) * 32, 16, 1024), C::IDESC_PV,
+                           (g > base || kk > 0) ? 1u : 0u);
+            } else {
+#pragma unroll
+              for (int kk = 0; kk < BN / 16; ++kk) {
+                umma_ts(tmem + C::COL_O, a + 8 * kk, sw128_desc(sV + kk * 2048, C::KBOX, 1024), C::IDESC_PV,
+                        (g > base || kk > 0) ? 1u : 0u);
+              }
             }
             tc_commit(b.v_empty0 + 8 * vs);   // V_g read, and O holds the item's tiles up to g
             tr(g, 4);
@@ -585,7 +614,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const float l_row = l_run + x_l[(half ^ 1) * BM + row];
       float sq = 0.f;
       if (live) {
-        const float inv = 1.f / l_row;
+        const float inv = (PV8 ? p.v_scale[head] : 1.f) / l_row;
         const int c0 = half * C::O_HALF;
         __nv_bfloat16* drow = dst + static_cast<size_t>(qrow) * D + head * HD + c0;
         const __nv_bfloat16* lrow = p.out_loc + static_cast<size_t>(qrow) * D + head * HD + c0;
@@ -623,7 +652,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       soft_barrier();
       if (row_ok && half == 0) {
         if (live && lse_dst)
-          lse_dst[static_cast<size_t>(head) * p.n_q + qrow] = (m_run + __log2f(l_row)) * 0.69314718055994531f;
+          lse_dst[static_cast<size_t>(head) * p.n_q + qrow] =
+              (m_run - C::P_SHIFT + __log2f(l_row)) * 0.69314718055994531f;
         if (with_disc)
           p.disc_part[static_cast<size_t>(head) * p.n_q + qrow] = x_sq[row] + x_sq[BM + row];
       }
@@ -664,6 +694,35 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           if (k & 1) acc1 = f2_add(acc1, f2_pack(e0, e1));
           else acc0 = f2_add(acc0, f2_pack(e0, e1));
           pk[k] = pack_bf16x2(e0, e1);
+        }
+        tmem_st4(pcol + 4 * c, pk);
+      }
+      const uint64_t acc = f2_add(acc0, acc1);
+      return __uint_as_float(static_cast<uint32_t>(acc)) + __uint_as_float(static_cast<uint32_t>(acc >> 32));
+    };
+    // PV8: P' = exp2(s * sl2 - m + P_SHIFT) as e4m3, four keys per TMEM column, this half's 96
+    // keys at key offset r + 96 * half of the tile's V window; returns the row-sum share of P'.
+    auto exps_store8 = [&](const uint32_t* s, float sl2, float m, uint32_t pcol) {
+      const float mm = m == -INFINITY ? 0.f : m;
+      const uint64_t negm = f2_pack(C::P_SHIFT - mm, C::P_SHIFT - mm);
+      const uint64_t sl2x2 = f2_pack(sl2, sl2);
+      uint64_t acc0 = 0, acc1 = 0;
+#pragma unroll
+      for (int c = 0; c < HALF_COLS / 16; ++c) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          float e[4];
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const int i = 16 * c + 4 * k + 2 * h2;
+            const uint64_t x = f2_fma(f2_pack(__uint_as_float(s[i]), __uint_as_float(s[i + 1])), sl2x2, negm);
+            e[2 * h2] = ex2_approx(__uint_as_float(static_cast<uint32_t>(x)));
+            e[2 * h2 + 1] = ex2_approx(__uint_as_float(static_cast<uint32_t>(x >> 32)));
+            if (h2) acc1 = f2_add(acc1, f2_pack(e[2], e[3]));
+            else acc0 = f2_add(acc0, f2_pack(e[0], e[1]));
+          }
+          pk[k] = pack_e4m3x4(e[0], e[1], e[2], e[3]);
         }
         tmem_st4(pcol + 4 * c, pk);
       }
@@ -752,7 +811,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         } else {
           // the running max stands unless the tile's max exceeds it by more than 2^8 somewhere in
           // the pair's rows (rare); then O is rescaled first
-          const bool need = ok && mx * sl2 > m_run + RESCALE_THRESHOLD;
+          const bool need = ok && mx * sl2 > m_run + C::RESCALE;
           if (pair_or(pair_id, need || !ok)) {
             float mo;
             ok = pair_exchange(mx, mo);
@@ -782,7 +841,21 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         if (threadIdx.x == 0) tr(g, 1);
         if (ok) {
-          l_run += exps_store(s, sl2, m_run, pcol);
+          if constexpr (PV8) {
+            // the tile's P V window starts at its first key rounded down to 16: P goes r keys in,
+            // with zeros before it (half 0) and after it up to the 224 keys the UMMAs read (half 1)
+            const int r4 = ((p.seg[seg].start + off) & 15) >> 2;
+            const uint32_t pbase = trow + C::COL_S0 + sb * BN;
+            l_run += exps_store8(s, sl2, m_run, pbase + r4 + 24 * half);
+            const uint32_t zero = 0u;
+            if (half == 0) {
+              for (int c = 0; c < r4; ++c) tmem_st1(pbase + c, &zero);
+            } else {
+              for (int c = 48 + r4; c < 8 * C::PV_STEPS; ++c) tmem_st1(pbase + c, &zero);
+            }
+          } else {
+            l_run += exps_store(s, sl2, m_run, pcol);
+          }
           if (threadIdx.x == 0) tr(g, 10);
           tmem_wait_st();
           tc_fence_before();
@@ -823,19 +896,20 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
 }
 
-template <int HD, bool QK8, bool TRACE = false>
+template <int HD, bool QK8, bool TRACE = false, bool PV8 = false>
 static cudaError_t launch_hd(const CUtensorMap* tq, const CUtensorMap* tkr, const CUtensorMap* tvr,
                              const CUtensorMap* tkc, const CUtensorMap* tvc, const AttnParams& p,
                              cudaStream_t s) {
-  using C = Cfg<HD, QK8>;
+  using C = Cfg<HD, QK8, PV8>;
   int dev = 0;
   cudaGetDevice(&dev);
   {
-    const cudaError_t e = set_smem_limit_once(reinterpret_cast<const void*>(attn_kernel<HD, QK8, TRACE>), C::SMEM);
+    const cudaError_t e =
+        set_smem_limit_once(reinterpret_cast<const void*>(attn_kernel<HD, QK8, PV8, TRACE>), C::SMEM);
     if (e != cudaSuccess) return e;
   }
   dim3 grid((p.n_q + BM - 1) / BM, p.num_heads);
-  attn_kernel<HD, QK8, TRACE><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
+  attn_kernel<HD, QK8, PV8, TRACE><<<grid, NTHREADS, C::SMEM, s>>>(*tq, *tkr, *tvr, *tkc, *tvc, p);
   return cudaGetLastError();
 }
 
@@ -843,6 +917,7 @@ cudaError_t launch_attention(int head_dim, const CUtensorMap* tq, const CUtensor
                              const CUtensorMap* tvr, const CUtensorMap* tkc,
                              const CUtensorMap* tvc, const AttnParams& p, cudaStream_t s) {
   if (p.q_scale) {
+    if (head_dim == 128 && p.v_scale) return launch_hd<128, true, false, true>(tq, tkr, tvr, tkc, tvc, p, s);
     if (head_dim == 128) return launch_hd<128, true>(tq, tkr, tvr, tkc, tvc, p, s);
     return cudaErrorInvalidValue;
   }

@@ -51,6 +51,8 @@ struct AttnParams {
   const float* q_scale;
   const float* kc_scale;
   const float* kr_scale;
+  // 8-bit P V (null for bf16 V): per-head e4m3 code scale of V (ring and chunk alike)
+  const float* v_scale;
 };
 
 // Raise the dynamic shared-memory limit of `func` to `bytes` on the current device, once
@@ -115,6 +117,10 @@ cudaError_t launch_quant_q_blocks(const void* x, int64_t n, int32_t H, int32_t d
                                   cudaStream_t s);
 cudaError_t launch_quant_given(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* q,
                                cudaStream_t s);
+// d-major e4m3 values: out[h][c][key] (key = t, or slots[t / P] * P + t % P when n_frames > 0);
+// d = 128, ld % 16 == 0, P % 4 == 0.
+cudaError_t launch_quant_vt(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* out,
+                            int64_t ld, int32_t P, int32_t n_frames, const int32_t* slots, cudaStream_t s);
 cudaError_t launch_append_qk8(const int32_t* slots, int32_t n_frames, int32_t P, int32_t H, int32_t d,
                               int64_t ring_tok, const void* k_src, const void* v_src, void* k_dst, void* v_dst,
                               const float* k_scale, cudaStream_t s);
@@ -136,6 +142,9 @@ bool encode_tmap_2d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1,
 // fp32 [d1][d0] with 128-byte swizzle (the Gram state, for bulk reduce-adds)
 bool encode_tmap_2d_f32(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
                         uint32_t b0, uint32_t b1);
+// uint8 (d0 inner, d1, d2) with 128-byte swizzle
+bool encode_tmap_3d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                       uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1, uint32_t b2);
 bool encode_tmap_2d_u8(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t stride1_bytes,
                        uint32_t b0, uint32_t b1);
 uint64_t wait_limit_ns();

@@ -14,7 +14,11 @@
 //       codes with given per-head scales (the chunk's keys with the ring's key scales).
 //   append_qk8_kernel
 //       appends frames to a ring whose keys are e4m3: K rows quantised with the ring's given
-//       per-head scales into their slots, V rows (bf16) copied.
+//       per-head scales into their slots, V rows (bf16) copied (or, for a ring whose values are
+//       e4m3 too, left to quant_vt_kernel).
+//   quant_vt_kernel
+//       values as d-major e4m3 codes [H][d][keys] with given per-head scales (the operand layout
+//       of the 8-bit P V): the chunk's values, or appended frames into their ring slots.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -176,7 +180,55 @@ __global__ void append_qk8_kernel(const AppendQk8Params p) {
     const int64_t dst_tok = static_cast<int64_t>(p.slot[f]) * p.P + tok % p.P;
     const int64_t dst = (static_cast<int64_t>(h) * p.ring_tok + dst_tok) * wpr + w;
     p.k_dst[dst] = quant8(p.k_src[i], inv_of_scale(p.k_scale[h]));
-    p.v_dst[dst] = p.v_src[i];
+    if (p.v_dst) p.v_dst[dst] = p.v_src[i];
+  }
+}
+
+// d-major e4m3 values: out[h][c][key(t)] = e4m3(v[t][h][c] * (1 / scale_h)), key(t) = t, or
+// slot[t / P] * P + t % P for appended frames.  One CTA per (block of 64 tokens, head): the block
+// is quantised into shared memory as [token][c], then written d-major, four consecutive tokens
+// (one 32-bit word: P % 4 == 0 keeps them in one frame and the word aligned) per store.
+constexpr int VT_TOK = 64;
+struct QuantVtParams {
+  const uint4* v;        // bf16 [n][H][d]
+  int64_t n;
+  int32_t H, d;
+  const float* scale;    // [H]
+  uint8_t* out;          // [H][d][ld]
+  int64_t ld;
+  int32_t P, n_frames;   // n_frames == 0: key(t) = t
+  int32_t slot[kMaxAppendFrames];
+};
+
+__global__ void __launch_bounds__(256) quant_vt_kernel(const QuantVtParams p) {
+  __shared__ __align__(16) uint8_t tile[VT_TOK][128 + 16];   // row padding spreads the d-major reads
+  const int h = blockIdx.y;
+  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * VT_TOK;
+  const int rows = static_cast<int>(p.n - t0 < VT_TOK ? p.n - t0 : VT_TOK);
+  const float inv = inv_of_scale(p.scale[h]);
+  const int wpr = p.d / 8;
+  for (int w = threadIdx.x; w < VT_TOK * wpr; w += blockDim.x) {
+    const int r = w / wpr, c8 = w % wpr;
+    uint2 code = make_uint2(0, 0);
+    if (r < rows) code = quant8(p.v[((t0 + r) * p.H + h) * wpr + c8], inv);
+    *reinterpret_cast<uint2*>(&tile[r][c8 * 8]) = code;
+  }
+  __syncthreads();
+  const int groups = (rows + 3) / 4;
+  for (int w = threadIdx.x; w < p.d * (VT_TOK / 4); w += blockDim.x) {
+    const int c = w / (VT_TOK / 4), g = w % (VT_TOK / 4);
+    if (g >= groups) continue;
+    const int r0 = 4 * g;
+    const int64_t t = t0 + r0;
+    const int64_t key = p.n_frames > 0 ? static_cast<int64_t>(p.slot[t / p.P]) * p.P + t % p.P : t;
+    uint8_t* dst = p.out + (static_cast<int64_t>(h) * p.d + c) * p.ld + key;
+    if (r0 + 3 < rows) {
+      *reinterpret_cast<uint32_t*>(dst) = static_cast<uint32_t>(tile[r0][c]) | (static_cast<uint32_t>(tile[r0 + 1][c]) << 8) |
+                                          (static_cast<uint32_t>(tile[r0 + 2][c]) << 16) |
+                                          (static_cast<uint32_t>(tile[r0 + 3][c]) << 24);
+    } else {
+      for (int i = 0; r0 + i < rows; ++i) dst[i] = tile[r0 + i][c];
+    }
   }
 }
 
@@ -224,6 +276,24 @@ cudaError_t launch_append_qk8(const int32_t* slots, int32_t n_frames, int32_t P,
   const int64_t total = static_cast<int64_t>(n_frames) * P * H * d / 8;
   const int64_t b = (total + 255) / 256;
   append_qk8_kernel<<<static_cast<unsigned>(b < sms * 8 ? b : sms * 8), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quant_vt(const void* x, int64_t n, int32_t H, int32_t d, const float* scale, uint8_t* out,
+                            int64_t ld, int32_t P, int32_t n_frames, const int32_t* slots, cudaStream_t s) {
+  QuantVtParams p{};
+  p.v = static_cast<const uint4*>(x);
+  p.n = n;
+  p.H = H;
+  p.d = d;
+  p.scale = scale;
+  p.out = out;
+  p.ld = ld;
+  p.P = P;
+  p.n_frames = n_frames;
+  for (int f = 0; f < n_frames; ++f) p.slot[f] = slots[f];
+  const dim3 grid(static_cast<unsigned>((n + VT_TOK - 1) / VT_TOK), static_cast<unsigned>(H));
+  quant_vt_kernel<<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();
 }
 

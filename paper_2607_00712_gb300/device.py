@@ -21,14 +21,22 @@ def to_f32(t: torch.Tensor) -> np.ndarray:
 class Ring:
     """A caller-owned KV ring: K and V [H][cap*P][d] tensors plus the C struct.
 
-    k_e4m3: keys as e4m3 codes (uint8), for the 8-bit query/key attention entry points."""
+    k_e4m3: keys as e4m3 codes (uint8), for the 8-bit query/key attention entry points.
+    kv_e4m3: keys as e4m3 codes and values as d-major e4m3 codes [H][d][vt_stride], for the
+    8-bit Q K^T and P V entry points."""
 
     def __init__(self, num_heads: int, head_dim: int, tokens_per_frame: int, capacity_frames: int,
-                 n_sink_frames: int = 0, device="cuda", k_e4m3: bool = False):
-        shape = (num_heads, capacity_frames * tokens_per_frame, head_dim)
-        self.k = torch.zeros(shape, dtype=torch.uint8 if k_e4m3 else torch.bfloat16, device=device)
-        self.v = torch.zeros(shape, dtype=torch.bfloat16, device=device)
-        self.c = KVRing(num_heads, head_dim, tokens_per_frame, capacity_frames, n_sink_frames, 1 if k_e4m3 else 0,
+                 n_sink_frames: int = 0, device="cuda", k_e4m3: bool = False, kv_e4m3: bool = False):
+        keys = capacity_frames * tokens_per_frame
+        shape = (num_heads, keys, head_dim)
+        fmt = 2 if kv_e4m3 else (1 if k_e4m3 else 0)
+        self.k = torch.zeros(shape, dtype=torch.uint8 if fmt else torch.bfloat16, device=device)
+        if kv_e4m3:
+            self.vt_stride = (keys + 15) // 16 * 16
+            self.v = torch.zeros(num_heads, head_dim, self.vt_stride, dtype=torch.uint8, device=device)
+        else:
+            self.v = torch.zeros(shape, dtype=torch.bfloat16, device=device)
+        self.c = KVRing(num_heads, head_dim, tokens_per_frame, capacity_frames, n_sink_frames, fmt,
                         0, self.k.data_ptr(), self.v.data_ptr())
 
     @property

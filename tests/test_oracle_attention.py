@@ -258,3 +258,14 @@ def test_frame_causal_needs_whole_frames():
     s = synth.make_step(17, 2, P, H, d, n_chunk_frames=2)
     with pytest.raises(ValueError):
         at.attn_full(s.q[:6], s.k_hist, s.v_hist, s.k_cur[:6], s.v_cur[:6], P, frame_causal=True)
+
+
+def test_attend_weights_are_the_softmax_of_attend():
+    # the weights reproduce attend's output and log-sum-exp (p V = O, max s + log L = LSE)
+    r = np.random.default_rng(31)
+    q, k, v = r.standard_normal((5, 8)), r.standard_normal((11, 8)), r.standard_normal((11, 3))
+    p, L = at.attend_weights(q, k, 0.4)
+    o, lse = at.attend(q, k, v, 0.4)
+    assert np.allclose(p.sum(axis=1), 1.0, atol=1e-14) and np.allclose(p @ v, o, atol=1e-13)
+    s = 0.4 * q @ k.T
+    assert np.allclose(s.max(axis=1) + np.log(L), lse, atol=1e-13) and np.all(L >= 1.0)
