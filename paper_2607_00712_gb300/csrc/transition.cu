@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactParams p) {
 // fp32, and *disc_sq_sum += sum_t disc[t]^2.  HBM-bound: one warp per token row, each lane
 // streaming 16-byte words of both rows with all its loads issued before the arithmetic.
 constexpr int DISC_WARPS = 8;
-constexpr int DISC_UNROLL = 4;
+constexpr int DISC_UNROLL = 8;   // 16-byte words per lane in flight per tensor: rows up to 2048 features in one pass
 
 __device__ __forceinline__ float sq_diff8(const uint4 a, const uint4 b) {
   const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
