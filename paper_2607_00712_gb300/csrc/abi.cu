@@ -330,14 +330,17 @@ ispa_status resolve(const ispa_kv_ring* r, ispa_window win, ispa_key_sets* ks) {
 // ------------------------------------------------------------ attention driver
 enum Mode { MODE_FULL, MODE_LOCAL, MODE_DUAL, MODE_HIST };
 
-int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P, int bn) {
+// align16: start every segment on a 16-key boundary (the d-major value tiles of the 8-bit P V
+// are TMA boxes whose first key must be a multiple of 16); the keys before the run are masked.
+int add_segs(AttnParams& p, int src, const ispa_slot_range* r, int n, int P, int bn, bool align16 = false) {
   int tiles = 0;
   for (int i = 0; i < n; ++i) {
     AttnSeg& s = p.seg[p.n_seg++];
     s.src = src;
-    s.start = r[i].first_slot * P;
-    s.count = r[i].n_slots * P;
-    s.pad = 0;
+    const int first = r[i].first_slot * P;
+    s.skip = align16 ? first & 15 : 0;
+    s.start = first - s.skip;
+    s.count = r[i].n_slots * P + s.skip;
     tiles += (s.count + bn - 1) / bn;
   }
   return tiles;
@@ -384,16 +387,17 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   const ispa_slot_range chunk{0, 0};
   (void)chunk;
   int tiles = 0;
+  const bool al = ring->k_format == ISPA_KV_KV_E4M3;
   if (mode == MODE_HIST) {
     // Eq. 10: the history set alone, no chunk
-    tiles = add_segs(p, 0, ks.hist, ks.n_hist, P, bn);
+    tiles = add_segs(p, 0, ks.hist, ks.n_hist, P, bn, al);
     if (tiles == 0) return launch_empty_branch(out, lse, n_q, H, HD, stream) == cudaSuccess ? ISPA_OK : ISPA_ERR_CUDA;
     p.n_local_tiles = tiles;
     p.n_tiles = tiles;
   } else if (mode == MODE_FULL) {
-    tiles += add_segs(p, 0, ks.full, ks.n_full, P, bn);
+    tiles += add_segs(p, 0, ks.full, ks.n_full, P, bn, al);
   } else {
-    tiles += add_segs(p, 0, ks.local, ks.n_local, P, bn);
+    tiles += add_segs(p, 0, ks.local, ks.n_local, P, bn, al);
   }
   if (mode != MODE_HIST) {
     AttnSeg& s = p.seg[p.n_seg++];
@@ -404,7 +408,7 @@ ispa_status attn_common(Mode mode, const ispa_kv_ring* ring, ispa_window win, co
   }
   if (mode != MODE_HIST) {
     p.n_local_tiles = tiles;
-    if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P, bn);
+    if (mode == MODE_DUAL) tiles += add_segs(p, 0, ks.hist, ks.n_hist, P, bn, al);
     p.n_tiles = tiles;
   }
   p.dual = mode == MODE_DUAL ? 1 : 0;

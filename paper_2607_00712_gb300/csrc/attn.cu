@@ -72,13 +72,13 @@ constexpr int P_HALF = HALF_COLS / 2;      // packed bf16 P columns per softmax 
 static_assert(BN % 16 == 0 && BN <= 256 && HALF_COLS % 8 == 0 && P_HALF % 4 == 0, "key tile shape");
 
 // PV8 (with QK8): V as e4m3 codes too, from d-major ("transposed") tiles [128 d rows][keys]: the
-// K-major B operand of a kind::f8f6f4 P V with P as e4m3 in TMEM.  A TMA box must start on a
-// 16-byte boundary, so a tile's V window starts at its first key rounded down to a multiple of
-// 16 and covers 256 keys (two 128-key boxes with 128-byte swizzle); P is written into TMEM
-// shifted by the remainder r, with zeros around it, and P V runs as 7 UMMAs of K = 32 over the
-// first 224 keys of the window (r + 192 <= 204).  P is scaled by 2^4 before its e4m3 rounding
-// (the running max is kept within 2^4 of every tile's max, so P' <= 2^8 < 448), which keeps
-// values down to 2^-10 of the row maximum in e4m3's normal range.
+// K-major B operand of a kind::f8f6f4 P V with P as e4m3 in TMEM (four keys per column).  A TMA
+// box must start on a 16-byte boundary, so every ring segment of this instance starts on a
+// 16-key boundary: the host moves its start back by up to 15 keys (`skip`), whose scores are
+// masked; a tile's V window is two 128-key boxes with 128-byte swizzle, and P V is 6 UMMAs of
+// K = 32.  P is scaled by 2^4 before its e4m3 rounding (the running max is kept within 2^4 of
+// every tile's max, so P' <= 2^8 < 448), which keeps values down to 2^-10 of the row maximum
+// in e4m3's normal range.
 // QK8: Q and K as e4m3 codes (one 128-byte swizzled row = the 128 features of a token), S by
 // kind::f8f6f4 UMMAs with K = 32; V, P and O as in the bf16 path.
 template <int HD, bool QK8 = false, bool PV8 = false>
@@ -92,7 +92,7 @@ struct Cfg {
   static constexpr int K_TILE = QK8 ? BN * HD : NBOX * KBOX;
   static constexpr int V_BOX8 = 128 * HD;                  // [HD rows][128 keys] e4m3 = 16 KB
   static constexpr int V_TILE = PV8 ? 2 * V_BOX8 : NBOX * KBOX;
-  static constexpr int PV_STEPS = PV8 ? 7 : BN / 16;       // UMMAs of one P V
+  static constexpr int PV_STEPS = PV8 ? BN / 32 : BN / 16;   // UMMAs of one P V
   static constexpr float RESCALE = PV8 ? 4.0f : RESCALE_THRESHOLD;   // lazy rescale bound (log2)
   static constexpr float P_SHIFT = PV8 ? 4.0f : 0.0f;      // log2 of the scale P gets before rounding
   static constexpr int KST = (HD == 128 && !QK8) ? 2 : 4;  // K stages
@@ -344,8 +344,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const uint32_t sV = sbase + C::OFF_V + vs * C::V_TILE;
         const int vhead = vk == kk ? kh : prev_h;
         if constexpr (PV8) {
-          // d-major e4m3 V: the 256-key window from the tile's first key rounded down to 16
-          const int x0 = (p.seg[vseg].start + voff) & ~15;
+          // d-major e4m3 V: the tile's first key is a multiple of 16 (segments start aligned)
+          const int x0 = p.seg[vseg].start + voff;
           tma_load_3d(sV, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, x0, 0, vhead);
           tma_load_3d(sV + C::V_BOX8, chunk ? &tm_vc : &tm_vr, b.v_full0 + 8 * vs, x0 + 128, 0, vhead);
         } else {
@@ -791,6 +791,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             for (int i = 0; i < HALF_COLS; ++i)
               if (i >= vloc) s[i] = __float_as_uint(-INFINITY);
           }
+          if constexpr (PV8) {
+            // keys before the run at the start of an aligned segment
+            const int vfirst = (off == 0 ? p.seg[seg].skip : 0) - half * HALF_COLS;
+            if (vfirst > 0) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i)
+                if (i < vfirst) s[i] = __float_as_uint(-INFINITY);
+            }
+          }
         };
         // P_j overwrites the first 96 columns of S_j (this half's 48 packed columns), so both
         // halves of the pair must have read their scores first: the pair barrier below orders it.
@@ -842,17 +851,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (threadIdx.x == 0) tr(g, 1);
         if (ok) {
           if constexpr (PV8) {
-            // the tile's P V window starts at its first key rounded down to 16: P goes r keys in,
-            // with zeros before it (half 0) and after it up to the 224 keys the UMMAs read (half 1)
-            const int r4 = ((p.seg[seg].start + off) & 15) >> 2;
-            const uint32_t pbase = trow + C::COL_S0 + sb * BN;
-            l_run += exps_store8(s, sl2, m_run, pbase + r4 + 24 * half);
-            const uint32_t zero = 0u;
-            if (half == 0) {
-              for (int c = 0; c < r4; ++c) tmem_st1(pbase + c, &zero);
-            } else {
-              for (int c = 48 + r4; c < 8 * C::PV_STEPS; ++c) tmem_st1(pbase + c, &zero);
-            }
+            // e4m3 P: this half's 96 keys are 24 columns of S_j's buffer
+            l_run += exps_store8(s, sl2, m_run, trow + C::COL_S0 + sb * BN + 24 * half);
           } else {
             l_run += exps_store(s, sl2, m_run, pcol);
           }

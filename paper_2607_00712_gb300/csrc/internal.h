@@ -18,7 +18,8 @@ struct AttnSeg {
   int32_t src;
   int32_t start;
   int32_t count;
-  int32_t pad;
+  int32_t skip;   // leading keys of the segment that are not in the key set (masked): 0, or the
+                  // alignment a segment of the 8-bit P V instance starts with
 };
 
 constexpr int kMaxSegs = 8;
