@@ -222,3 +222,25 @@ def test_minimum_sizes_one_query_one_head(d):
     st = Step(51, P=1, H=1, d=d, n_past=5, n_chunk_frames=1, capacity=3, n_sink_pinned=1)
     assert st.n_q == 1
     _check_all_modes(st, (1, 1))
+
+
+def test_work_stealing_covers_every_item():
+    # 64 heads x 5 query tiles = 320 (query tile, head) items, about twice the SM count: the
+    # CTAs that start first take the items of CTAs that have not started (cluster launch
+    # control).  Every row of every item is checked against the oracle, and repeated calls
+    # must agree bit for bit whichever CTA ran an item.
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    st = Step(61, P=128, H=64, d=128, n_past=3, n_chunk_frames=5, capacity=4)
+    assert st.n_q == 640 and 5 * st.H > n_sm
+    o, l = _run_full(st)
+    ro, rl = at.attn_full(*st.oracle_args())
+    assert_close_attn(o, ro, "stolen items full")
+    assert np.abs(l - rl).max() < 2e-3
+    for _ in range(3):
+        o2, l2 = _run_full(st)
+        assert np.array_equal(o2, o) and np.array_equal(l2, l)
+    g = _run_dual(st, (0, 1))
+    r = at.attn_dual(*st.oracle_args(), 0, 1)
+    assert_close_attn(g["a_full"], r["a_full"], "stolen items dual full")
+    assert_close_attn(g["a_loc"], r["a_loc"], "stolen items dual loc")
+    assert_disc_close(g["a_full"], g["a_loc"], g["disc"], r, "stolen items disc", g["disc_sum"])
