@@ -28,7 +28,9 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include "delta.cuh"
 #include "internal.h"
+#include "pdl.cuh"
 #include "ptx.cuh"
 
 namespace ispa {
@@ -166,23 +168,10 @@ __global__ void __launch_bounds__(256) split_kernel(const uint4* __restrict__ a_
                                                     const uint4* __restrict__ a_full,
                                                     uint4* __restrict__ hi, uint4* __restrict__ lo,
                                                     int64_t n_words) {
+  pdl_trigger();   // the Gram kernel after this one may set itself up meanwhile
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
-    const uint4 a = a_loc[i], f = a_full[i];
-    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
-    uint32_t hw[4], lw[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float d0 = __uint_as_float(fw[e] << 16) - __uint_as_float(aw[e] << 16);
-      const float d1 = __uint_as_float(fw[e] & 0xFFFF0000u) - __uint_as_float(aw[e] & 0xFFFF0000u);
-      const uint32_t h = pack_bf16x2(d0, d1);
-      const float h0 = __uint_as_float(h << 16), h1 = __uint_as_float(h & 0xFFFF0000u);
-      hw[e] = h;
-      lw[e] = pack_bf16x2(d0 - h0, d1 - h1);
-    }
-    hi[i] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-    lo[i] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-  }
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride)
+    split_delta8(a_loc[i], a_full[i], hi[i], lo[i]);
 }
 
 template <int BN>
@@ -234,6 +223,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();   // the operands and the state may come from the kernel before this one
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
 
   if (warp == 0) {
@@ -510,6 +500,7 @@ __global__ void __launch_bounds__(W_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();   // the operands and the state may come from the kernel before this one
   const WaitCtx wc{abort_flag, p.status, p.wait_limit_ns};
 
   if (warp == 0) {
@@ -684,8 +675,7 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   p.status = status;
   p.wait_limit_ns = wait_limit_ns;
   p.heartbeat = hb;
-  gram_wide_kernel<<<grid, W_THREADS, W_SMEM, s>>>(tm[0], tm[1], tm[2], tm_state, p);
-  return cudaGetLastError();
+  return launch_pdl(gram_wide_kernel, grid, dim3(W_THREADS), W_SMEM, s, tm[0], tm[1], tm[2], tm_state, p);
 }
 
 size_t ls_accumulate_ws_bytes(int32_t D, int64_t T) {
@@ -735,8 +725,8 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   // one CTA per SM, each with at least 16 steps (a 1024-token run of one tile)
   const int64_t want = (total + 15) / 16;
   const dim3 grid(static_cast<unsigned>(want < sms ? (want > 0 ? want : 1) : sms));
-  gram_kernel<BN><<<grid, G_THREADS, C::SMEM, s>>>(tr[0], tr[1], tr[2], tc[0], tc[1], tc[2], p);
-  return cudaGetLastError();
+  return launch_pdl(gram_kernel<BN>, grid, dim3(G_THREADS), C::SMEM, s, tr[0], tr[1], tr[2], tc[0], tc[1], tc[2],
+                    p);
 }
 
 cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full, void* ws,
@@ -756,6 +746,11 @@ cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const 
       reinterpret_cast<uint4*>(lo), n_words);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  return launch_ls_gram(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
+}
+
+cudaError_t launch_ls_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo, float* gram,
+                           int* status, uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
   if (D % 256 == 0) return launch_gram_wide(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
   return launch_gram<128>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
 }

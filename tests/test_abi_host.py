@@ -156,6 +156,28 @@ def test_attention_option_validation_without_gpu():
                                16, 1 << 20, None) == abi.ISPA_ERR_INVALID_ARG
 
 
+def test_delta_entry_points_validation_without_gpu():
+    L = abi.lib()
+    r = KVRing(2, 64, 16, 4, 0, 0, 2, 16, 16)
+    # ring, win, q, k_cur, v_cur, n_q, scale, flags, a_full, a_loc, hi, lo, disc, dsum, lse x2, ws, ws_bytes
+    args = [ctypes.byref(r), Window(0, 1), 16, 16, 16, 32, 0.0, 0, 16, 16, 16, 16, 16, 16, None, None, 16, 1 << 20,
+            None]
+    for i, bad in [(10, None), (11, None), (10, 18), (11, 24)]:   # a missing or misaligned hi / lo
+        a = list(args)
+        a[i] = bad
+        assert L.ispa_attn_dual_delta(*a) == abi.ISPA_ERR_INVALID_ARG, (i, bad)
+    a = list(args)
+    a[16] = None
+    assert L.ispa_attn_dual_delta(*a) == abi.ISPA_ERR_WORKSPACE
+    st = LSState(100, 0, 0, 16)
+    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, 16, 10, None) == abi.ISPA_ERR_UNSUPPORTED
+    st = LSState(128, 0, 0, 16)
+    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, 16, 0, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 24, 16, 10, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, None, 10, None) == abi.ISPA_ERR_INVALID_ARG
+    assert st.n_tokens == 0
+
+
 def test_w8a8_validation_without_gpu():
     L = abi.lib()
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 100, 192, 256, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D % 128

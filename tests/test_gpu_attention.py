@@ -244,3 +244,39 @@ def test_work_stealing_covers_every_item():
     assert_close_attn(g["a_full"], r["a_full"], "stolen items dual full")
     assert_close_attn(g["a_loc"], r["a_loc"], "stolen items dual loc")
     assert_disc_close(g["a_full"], g["a_loc"], g["disc"], r, "stolen items disc", g["disc_sum"])
+
+
+def test_repeated_launches_at_the_step_shape_are_bit_identical():
+    # 444 items at the 1.3B step shape, each launch redistributing them over the SMs by work
+    # stealing: 12 rounds of the three modes launched back to back on one stream, with no host
+    # synchronisation between them, must reproduce the first launches' outputs bit for bit (the
+    # arithmetic of an item does not depend on which CTA runs it, and no item may be skipped or
+    # run twice)
+    st = Step(62, P=1560, H=12, d=128, n_past=18, n_chunk_frames=3, capacity=18)
+    D = st.H * st.d
+    ref_f, _ = _run_full(st)
+    ref_l, _ = _run_local(st, (0, 6))
+    g = _run_dual(st, (0, 6))
+    wsb = abi.ispa_attn_dual_workspace_size(st.H, st.n_q)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+    rounds = []
+    for _ in range(12):
+        outs = [torch.empty(st.n_q, D, dtype=torch.bfloat16, device="cuda") for _ in range(4)]
+        disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+        abi.ispa_attn_full(st.ring.c, st.q, st.kc, st.vc, st.n_q, 0.0, outs[0])
+        abi.ispa_attn_local(st.ring.c, Window(0, 6), st.q, st.kc, st.vc, st.n_q, 0.0, outs[1])
+        abi.ispa_attn_dual(st.ring.c, Window(0, 6), st.q, st.kc, st.vc, st.n_q, 0.0, outs[2], outs[3], disc, dsum,
+                           None, None, ws, wsb)
+        rounds.append((outs, disc))
+    torch.cuda.synchronize()
+    assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
+    bad = []
+    for i, (outs, disc) in enumerate(rounds):
+        for name, t, ref in [("full", outs[0], ref_f), ("local", outs[1], ref_l), ("dual full", outs[2], g["a_full"]),
+                             ("dual loc", outs[3], g["a_loc"])]:
+            if not np.array_equal(to_f32(t).reshape(ref.shape), ref):
+                bad.append((i, name))
+        if not np.array_equal(to_f32(disc), g["disc"]):
+            bad.append((i, "disc"))
+    assert not bad, bad
