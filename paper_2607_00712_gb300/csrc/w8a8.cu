@@ -12,8 +12,8 @@
 // oracle's): amax = max |x|; inv = 448 / amax, scale = amax / 448 (both 1 for an all-zero
 // group); code = e4m3(x * inv), round to nearest even with saturation at +-448.
 //
-// GEMM: persistent, one CTA per SM looping over 128 x BN output tiles (BN = 256 when
-// D_out % 256 == 0 and there are at least two waves of such tiles, else 128); both operands
+// GEMM: persistent, one CTA per SM looping over 128 x BN output tiles (BN = 256, 192 or 128,
+// whichever gives the shortest estimated run: waves of tiles x their cost); both operands
 // K-major with 128-byte swizzle (one 128-byte row = 128 codes = four K=32 UMMA steps), a
 // 4-stage TMA ring that runs on across tile boundaries, two accumulator sets in TMEM so that
 // the epilogue of one tile (both scales, bf16 store) overlaps the UMMAs of the next; with
@@ -23,6 +23,8 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
+
+#include <algorithm>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -161,12 +163,13 @@ template <int BN>
 struct QCfg {
   // Persistent: one CTA per SM loops over output tiles.  Two accumulator sets in TMEM let the
   // epilogue of one tile overlap the UMMAs of the next; with 128-column tiles each set holds
-  // two accumulation chains (k-steps alternate between them), with 256-column tiles one.
-  static constexpr int CHAINS = BN == 256 ? 1 : 2;
+  // two accumulation chains (k-steps alternate between them), with 192- and 256-column tiles one.
+  static_assert(BN == 128 || BN == 192 || BN == 256, "tile width");
+  static constexpr int CHAINS = BN == 128 ? 2 : 1;
   static constexpr int SET = CHAINS * BN;         // TMEM columns per accumulator set
   static constexpr int QST = 4;
   static constexpr int A_BYTES = QM * QK;         // 16 KB
-  static constexpr int B_BYTES = BN * QK;         // 32 or 16 KB
+  static constexpr int B_BYTES = BN * QK;         // 32, 24 or 16 KB
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int OFF_BAR = QST * STAGE;
   static constexpr int N_BAR = 2 * QST + 4 + 1;   // full/empty per stage, set full/empty x2, drain
@@ -175,8 +178,8 @@ struct QCfg {
   // allocation never waits for another CTA
   static_assert(SMEM > 116 * 1024 && SMEM <= 232448 && STAGE % 1024 == 0, "shared memory layout");
   static constexpr uint32_t IDESC = idesc_e4m3(QM, BN);
-  static constexpr uint32_t TMEM_COLS = 2 * SET;
-  static_assert(TMEM_COLS == 512, "two accumulator sets fill TMEM");
+  static constexpr uint32_t TMEM_COLS = 512;      // the allocation (a power of two)
+  static_assert(2 * SET <= 512, "two accumulator sets fit in TMEM");
 };
 
 struct GemmParams {
@@ -402,11 +405,28 @@ cudaError_t launch_w8a8_gemm(const uint8_t* a_q, const float* a_scale, const uin
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // 256-column tiles halve the activation re-reads, but with under two waves of them the
-  // last partial wave leaves SMs idle for a large share of the run: then take 128-column tiles
-  const int64_t tiles256 = static_cast<int64_t>((T + QM - 1) / QM) * (Dout / 256);
-  if (Dout % 256 == 0 && tiles256 >= 2 * static_cast<int64_t>(sms))
+  // Estimated run: waves of tiles (one tile per SM per wave) x the time of one tile.  A
+  // k-block of a 128 x BN tile moves (128 + BN) x 128 bytes through shared memory twice (TMA
+  // write, UMMA read) for 128 x BN x 128 MACs, so wider tiles need fewer bytes per MAC: relative
+  // time per tile at the shared-memory limit ~ (128 + BN), with a floor at the tensor rate.
+  const int64_t m_tiles = (T + QM - 1) / QM;
+  int best = 128;
+  double best_cost = 0.0;
+  for (const int bn : {256, 192, 128}) {
+    if (Dout % bn != 0) continue;
+    const int64_t tiles = m_tiles * (Dout / bn);
+    const double waves = static_cast<double>((tiles + sms - 1) / sms);
+    const double per_tile = std::max(static_cast<double>(128 + bn), 1.5 * bn);
+    const double cost = waves * per_tile;
+    if (best_cost == 0.0 || cost < best_cost) {
+      best = bn;
+      best_cost = cost;
+    }
+  }
+  if (best == 256)
     return launch_gemm_bn<256>(a_q, a_scale, w_q, w_scale, T, D, Dout, o, status, wait_limit_ns, s);
+  if (best == 192)
+    return launch_gemm_bn<192>(a_q, a_scale, w_q, w_scale, T, D, Dout, o, status, wait_limit_ns, s);
   return launch_gemm_bn<128>(a_q, a_scale, w_q, w_scale, T, D, Dout, o, status, wait_limit_ns, s);
 }
 

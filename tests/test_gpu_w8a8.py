@@ -103,10 +103,11 @@ def test_quantize_weight_bit_exact(with_dw):
     assert np.array_equal(s.cpu().numpy(), rs)
 
 
-@pytest.mark.parametrize("T,D,Do", [(300, 256, 384), (300, 256, 512), (77, 384, 256), (130, 128, 128)])
-def test_linear_ragged_and_both_tile_widths(T, D, Do):
-    # D_out = 384 and 128 take the 128-column tile, 512 and 256 the 256-column tile;
-    # T leaves a ragged last row tile
+@pytest.mark.parametrize("T,D,Do", [(300, 256, 384), (300, 256, 512), (77, 384, 256), (130, 128, 128),
+                                    (4611, 256, 1536)])
+def test_linear_ragged_and_every_tile_width(T, D, Do):
+    # D_out = 384 and 128 take the 128-column tile, 512 and 256 the 256-column tile, and 1536
+    # with 37 row tiles the 192-column tile (296 tiles: two waves); T leaves a ragged last row tile
     x = _activations(4, T, D)
     W = synth.make_weight(5, D, Do)
     aq, sa = _gpu_quant_rows(x)
