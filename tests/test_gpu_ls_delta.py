@@ -149,3 +149,67 @@ def test_dual_delta_chain_equals_two_input_chain_at_the_step_shape():
     for (n1, b1), b2 in zip(zip("GXS", ls1.blocks()), ls2.blocks()):
         assert _rel(b1, b2) <= 1e-6, n1
     assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
+
+
+def test_dual_delta_frame_causal_matches_dual_ex():
+    # the option bits pass through: frame-causal chunk in both outputs, the pair from them
+    st = Step(64, P=96, H=2, d=128, n_past=5, n_chunk_frames=3, capacity=8)
+    D = st.H * st.d
+    bf = torch.bfloat16
+    outs = {}
+    for name in ("ex", "delta"):
+        a_full = torch.empty(st.n_q, D, dtype=bf, device="cuda")
+        a_loc = torch.empty(st.n_q, D, dtype=bf, device="cuda")
+        disc = torch.empty(st.n_q, dtype=torch.float32, device="cuda")
+        dsum = torch.zeros(1, dtype=torch.float32, device="cuda")
+        wsb = abi.ispa_attn_dual_workspace_size(st.H, st.n_q)
+        ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+        if name == "ex":
+            abi.ispa_attn_dual_ex(st.ring.c, Window(0, 2), st.q, st.kc, st.vc, st.n_q, 0.0, abi.ISPA_ATTN_FRAME_CAUSAL,
+                                  a_full, a_loc, disc, dsum, None, None, ws, wsb)
+            outs[name] = (a_full, a_loc, disc)
+        else:
+            hi = torch.empty(st.n_q, D, dtype=bf, device="cuda")
+            lo = torch.empty(st.n_q, D, dtype=bf, device="cuda")
+            abi.ispa_attn_dual_delta(st.ring.c, Window(0, 2), st.q, st.kc, st.vc, st.n_q, 0.0,
+                                     abi.ISPA_ATTN_FRAME_CAUSAL, a_full, a_loc, hi, lo, disc, dsum, None, None, ws, wsb)
+            outs[name] = (a_full, a_loc, disc, hi, lo)
+    torch.cuda.synchronize()
+    for a, b in zip(outs["ex"], outs["delta"][:3]):
+        assert np.array_equal(a.cpu().view(torch.int32 if a.dtype == torch.float32 else torch.int16).numpy(),
+                              b.cpu().view(torch.int32 if b.dtype == torch.float32 else torch.int16).numpy())
+    hi, lo = _split_host(to_f32(outs["delta"][1]), to_f32(outs["delta"][0]))
+    assert np.array_equal(_bits(outs["delta"][3]), _bits(hi)) and np.array_equal(_bits(outs["delta"][4]), _bits(lo))
+
+
+@pytest.mark.parametrize("D", [384, 1536])
+def test_back_to_back_accumulates_in_both_forms(D):
+    # Six accumulate calls on one stream with no host synchronisation, alternating the two-input
+    # and the pre-split form: each Gram launch starts under the end of the kernel before it and
+    # must see the state the previous Gram launch wrote.
+    st = LS(D)
+    ref = ols.ls_state(D)
+    bufs = []
+    for i in range(6):
+        T = [700, 64, 1313, 5, 2048, 999][i]
+        a_loc, a_full = synth.make_activations(9100 + 17 * i + D, T, D)
+        ols.ls_accumulate(ref, a_loc, a_full)
+        a_d, f_d = bf16_tensor(a_loc), bf16_tensor(a_full)
+        if i % 2:
+            hi, lo = _split_host(a_loc, a_full)
+            hi, lo = hi.cuda(), lo.cuda()
+            bufs.append((a_d, hi, lo))
+            abi.ispa_ls_accumulate_delta(st.c, a_d, hi, lo, T)
+        else:
+            wsb = abi.ispa_ls_accumulate_workspace_size(D, T)
+            ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+            bufs.append((a_d, f_d, ws))
+            abi.ispa_ls_accumulate(st.c, a_d, f_d, T, ws, wsb)
+    torch.cuda.synchronize()
+    assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
+    full = st.gram.view(2 * D, 2 * D).double().cpu().numpy()
+    G, X, S = full[:D, :D], full[:D, D:], full[D:, D:]
+    keep = _maintained_mask(D)
+    assert _rel(G[keep], ref["G"][keep]) <= 1e-3
+    assert _rel(S[keep], ref["S"][keep]) <= 1e-3
+    assert _rel(X, ref["X"]) <= 1e-3
