@@ -324,11 +324,13 @@ class StepRunner:
         """The step's result tensors (the ones an e2e run reads back)."""
         return [self.out_full, self.out_local, self.a_full, self.a_loc, self.disc]
 
-    def step(self, ev=None, inputs=None, outs=None):
+    def step(self, ev=None, inputs=None, outs=None, in_events=None):
         """Enqueue one step; ev = list of 6 events to record between the calls (or None).
 
         inputs / outs: another set of (q, k_cur, v_cur) triples / result tensors of the same
-        shapes (the e2e pipeline alternates two sets); default: the runner's own."""
+        shapes (the e2e pipeline alternates two sets); default: the runner's own.
+        in_events: one event per layer, recorded once that layer's inputs are on the device;
+        the layer's attention call waits for its own (or None)."""
         abi, nq = self.abi, self.wl["nq"]
         s = self.stream
         inputs = self.inputs if inputs is None else inputs
@@ -340,13 +342,17 @@ class StepRunner:
                 log(f"[bench]   call {i} done, device status {st}/{code}")
         else:
             rec = (lambda i: ev[i].record(s)) if ev else (lambda i: None)
+        wait_in = (lambda k: s.wait_event(in_events[k])) if in_events else (lambda k: None)
         rec(0)
+        wait_in(0)
         q, kc, vc = inputs[0]
         abi.ispa_attn_full(self.rings[0].c, q, kc, vc, nq, 0.0, out_full, None, s)
         rec(1)
+        wait_in(1)
         q, kc, vc = inputs[1]
         abi.ispa_attn_local(self.rings[1].c, self.win, q, kc, vc, nq, 0.0, out_local, None, s)
         rec(2)
+        wait_in(2)
         q, kc, vc = inputs[2]
         abi.ispa_attn_dual_delta(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, 0, a_full, a_loc, self.delta_hi,
                                  self.delta_lo, disc, self.disc_sum, None, None, self.dual_ws, self.dual_wsb, s)
@@ -967,9 +973,10 @@ def run_e2e(r, args, device, flops_step, world):
     Every step copies its own inputs host->device before its compute and reads its results
     device->host after it.  The copies of step i+1 (in) and i-1 (out) run on two copy streams
     while step i computes: two sets of device inputs and outputs alternate, ordered by events
-    (step i's inputs land before it starts; a set is refilled only after the step that used it
-    has finished computing and has been read back).  Timed from the first copy in to the last
-    copy out, divided by the number of steps.
+    (each layer's call waits for that layer's inputs, each result is read back once the call
+    that writes it has finished; a set is refilled only after the step that used it has finished
+    computing and has been read back).  Timed from the first copy in to the last copy out,
+    divided by the number of steps.
     """
     import torch
     host_in = [[t.cpu().pin_memory() for t in trip] for trip in r.inputs]
@@ -986,6 +993,7 @@ def run_e2e(r, args, device, flops_step, world):
         ev_comp, ev_out = [], []
         for i in range(steps):
             b = i % 2
+            e_in = []
             with torch.cuda.stream(s_in):
                 if i >= 2:
                     s_in.wait_event(ev_comp[i - 2])          # set b no longer read by step i-2
@@ -994,18 +1002,18 @@ def run_e2e(r, args, device, flops_step, world):
                 for trip_h, trip_d in zip(host_in, dev_in[b]):
                     for h, dv in zip(trip_h, trip_d):
                         dv.copy_(h, non_blocking=True)
-                e_in = torch.cuda.Event()
-                e_in.record(s_in)
-            s_comp.wait_event(e_in)
+                    e = torch.cuda.Event()
+                    e.record(s_in)                           # this layer's inputs are in
+                    e_in.append(e)
             if i >= 2:
                 s_comp.wait_event(ev_out[i - 2])             # outputs of set b read back
-            r.step(inputs=dev_in[b], outs=dev_out[b])
-            e_c = torch.cuda.Event()
-            e_c.record(s_comp)
-            ev_comp.append(e_c)
+            ev = [torch.cuda.Event() for _ in range(6)]
+            r.step(ev=ev, inputs=dev_in[b], outs=dev_out[b], in_events=e_in)
+            ev_comp.append(ev[5])
             with torch.cuda.stream(s_out):
-                s_out.wait_event(e_c)
-                for h, dv in zip(host_out, dev_out[b]):
+                # out_full after the F call, out_local after L, a_full, a_loc, disc after the dual
+                for h, dv, k in zip(host_out, dev_out[b], (1, 2, 3, 3, 3)):
+                    s_out.wait_event(ev[k])
                     h.copy_(dv, non_blocking=True)
                 e_o = torch.cuda.Event()
                 e_o.record(s_out)
