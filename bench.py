@@ -97,16 +97,18 @@ def roofline_entry(model, achieved, pk):
                 frac_of_nominal=round(achieved / NOMINAL_BF16_TFLOPS, 4), nominal_peak=NOMINAL_BF16_TFLOPS)
 
 
-def ls_flops(D, T):
+def ls_flops(D, T, exact=False):
     """FLOPs of one LS accumulation: the method's own work (the upper triangles of G = A^T A and
     S = Delta^T Delta with their diagonals, and all of X = A^T Delta: 2 T (2 D^2 + D)) and the
-    tile work the kernel issues (256 x 256 tiles with whole diagonal tiles; X in two passes and S
-    in three over the bf16 hi/lo split of Delta, or 128 x 128 tiles when D % 256 != 0)."""
+    tile work the kernel issues (256 x 256 tiles with whole diagonal tiles, or 128 x 128 when
+    D % 256 != 0; one pass per tile in the default scaled form, X in two passes and S in three
+    over the bf16 hi/lo split of Delta in the exact form)."""
     method = 2.0 * T * (2.0 * D * D + D)
     tb = 256 if D % 256 == 0 else 128
     nb = D // tb
     upper = nb * (nb + 1) // 2
-    tile = (upper + 2 * nb * nb + 3 * upper) * 2.0 * tb * tb * T
+    passes = (1, 2, 3) if exact else (1, 1, 1)
+    tile = (passes[0] * upper + passes[1] * nb * nb + passes[2] * upper) * 2.0 * tb * tb * T
     return method, tile
 
 
@@ -309,15 +311,12 @@ class StepRunner:
         self.disc_sum = torch.zeros(1, dtype=torch.float32, device=device)
         self.dual_wsb = abi.ispa_attn_dual_workspace_size(H, nq)
         self.dual_ws = torch.empty(self.dual_wsb, dtype=torch.uint8, device=device)
-        # Delta = A_full - A_loc as the bf16 hi / lo pair the dual pass writes for the LS sums
-        self.delta_hi = torch.empty(nq, D, dtype=bf, device=device)
-        self.delta_lo = torch.empty(nq, D, dtype=bf, device=device)
         self.ls = LS(D, device)
         self.ls_wsb = abi.ispa_ls_accumulate_workspace_size(D, nq)
         self.ls_ws = torch.empty(self.ls_wsb, dtype=torch.uint8, device=device)
         self.ring_arr = (abi.KVRing * 3)()
         self.stream = torch.cuda.current_stream(device)
-        self.launches_per_step = 6   # 3 attention + disc reduce + gram + append
+        self.launches_per_step = 8   # 3 attention + disc reduce + amax + convert + gram + append
         torch.cuda.synchronize(device)
 
     def outputs(self):
@@ -354,10 +353,10 @@ class StepRunner:
         rec(2)
         wait_in(2)
         q, kc, vc = inputs[2]
-        abi.ispa_attn_dual_delta(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, 0, a_full, a_loc, self.delta_hi,
-                                 self.delta_lo, disc, self.disc_sum, None, None, self.dual_ws, self.dual_wsb, s)
+        abi.ispa_attn_dual(self.rings[2].c, self.win, q, kc, vc, nq, 0.0, a_full, a_loc, disc,
+                           self.disc_sum, None, None, self.dual_ws, self.dual_wsb, s)
         rec(3)
-        abi.ispa_ls_accumulate_delta(self.ls.c, a_loc, self.delta_hi, self.delta_lo, nq, s)
+        abi.ispa_ls_accumulate(self.ls.c, a_loc, a_full, nq, self.ls_ws, self.ls_wsb, s)
         rec(4)
         for i in range(3):
             self.ring_arr[i] = self.rings[i].c
@@ -606,35 +605,26 @@ def run_extras(r, wl, device, reps=20):
         if i >= 3:
             t_disc += ev[0].elapsed_time(ev[1])
     t_disc /= reps
-    # the warmup layer's dual + LS chain in both forms, L2 flushed before each: the two-input LS
-    # call (its own pass forms and splits Delta from A_loc and A_full) against the dual pass
-    # that writes the split pair itself (the step's form)
-    ev6 = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
-    t_ch = np.zeros(4)
+    # LS accumulate in its exact form (Delta as a bf16 hi / lo pair) against the default scaled
+    # form on the same inputs, L2 flushed before each
+    ev6 = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    t_ls = np.zeros(2)
     for i in range(reps + 3):
         flush.fill_(float(i))
         ev6[0].record(s)
-        abi.ispa_attn_dual(ring, r.win, q, kc, vc, nq, 0.0, r.a_full, r.a_loc, r.disc, r.disc_sum, None, None,
-                           r.dual_ws, r.dual_wsb, s)
-        ev6[1].record(s)
         abi.ispa_ls_accumulate(r.ls.c, r.a_loc, r.a_full, nq, r.ls_ws, r.ls_wsb, s)
-        ev6[2].record(s)
+        ev6[1].record(s)
         flush.fill_(float(i) + 0.5)
+        ev6[2].record(s)
+        abi.ispa_ls_accumulate_ex(r.ls.c, r.a_loc, r.a_full, nq, abi.ISPA_LS_EXACT_DELTA, r.ls_ws, r.ls_wsb, s)
         ev6[3].record(s)
-        abi.ispa_attn_dual_delta(ring, r.win, q, kc, vc, nq, 0.0, 0, r.a_full, r.a_loc, r.delta_hi, r.delta_lo,
-                                 r.disc, r.disc_sum, None, None, r.dual_ws, r.dual_wsb, s)
-        ev6[4].record(s)
-        abi.ispa_ls_accumulate_delta(r.ls.c, r.a_loc, r.delta_hi, r.delta_lo, nq, s)
-        ev6[5].record(s)
         torch.cuda.synchronize(device)
         if i >= 3:
-            t_ch += [ev6[0].elapsed_time(ev6[1]), ev6[1].elapsed_time(ev6[2]), ev6[3].elapsed_time(ev6[4]),
-                     ev6[4].elapsed_time(ev6[5])]
-    t_ch /= reps
-    out.update(two_input_chain=dict(dual_ms=round(t_ch[0], 4), ls_accumulate_ms=round(t_ch[1], 4),
-                                    total_ms=round(t_ch[0] + t_ch[1], 4)),
-               delta_chain=dict(dual_delta_ms=round(t_ch[2], 4), ls_accumulate_delta_ms=round(t_ch[3], 4),
-                                total_ms=round(t_ch[2] + t_ch[3], 4)))
+            t_ls += [ev6[0].elapsed_time(ev6[1]), ev6[2].elapsed_time(ev6[3])]
+    t_ls /= reps
+    _, tile_exact = ls_flops(D, nq, exact=True)
+    out.update(ls_accumulate_scaled_ms=round(t_ls[0], 4), ls_accumulate_exact_ms=round(t_ls[1], 4),
+               ls_exact_tile_tflops=round(tile_exact / (t_ls[1] * 1e-3) / 1e12, 1))
     disc_bytes = 2 * nq * D * 2 + nq * 4
     pk = peaks()
     out.update(discrepancy_ms=round(t_disc, 4), discrepancy_gbs=round(disc_bytes / (t_disc * 1e-3) / 1e9, 1),
@@ -931,8 +921,8 @@ def run_warmup(wl, device, steps=8, cache_frames=24):
     dsum = torch.zeros(1, dtype=torch.float32, device=device)
     wsb = abi.ispa_attn_dual_workspace_size(H, nq)
     ws = torch.empty(wsb, dtype=torch.uint8, device=device)
-    hi = torch.empty_like(a_full)
-    lo = torch.empty_like(a_full)
+    lwsb = abi.ispa_ls_accumulate_workspace_size(D, nq)
+    lws = torch.empty(lwsb, dtype=torch.uint8, device=device)
     qkv = [_device_qkv(g, L, P, H, d) for _ in range(steps)]
     s = torch.cuda.current_stream(device)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
@@ -940,10 +930,9 @@ def run_warmup(wl, device, steps=8, cache_frames=24):
     torch.cuda.synchronize(device)
     for q, kc, vc in qkv:
         ev[0].record(s)
-        abi.ispa_attn_dual_delta(ring.c, win, q, kc, vc, nq, 0.0, 0, a_full, a_loc, hi, lo, disc, dsum, None, None,
-                                 ws, wsb, s)
+        abi.ispa_attn_dual(ring.c, win, q, kc, vc, nq, 0.0, a_full, a_loc, disc, dsum, None, None, ws, wsb, s)
         ev[1].record(s)
-        abi.ispa_ls_accumulate_delta(st.c, a_loc, hi, lo, nq, s)
+        abi.ispa_ls_accumulate(st.c, a_loc, a_full, nq, lws, lwsb, s)
         ev[2].record(s)
         torch.cuda.synchronize(device)
         t_dual += ev[0].elapsed_time(ev[1])

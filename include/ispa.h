@@ -344,28 +344,6 @@ ISPA_API ispa_status ispa_attn_dual_ex(const ispa_kv_ring* ring, ispa_window win
                               float* disc_sq_sum, float* lse_full, float* lse_loc, void* workspace,
                               size_t ws_bytes, ispa_stream stream);
 
-/*
- * ispa_attn_dual (with option bits, as ispa_attn_dual_ex) that also writes the
- * difference of its two outputs in the form ispa_ls_accumulate_delta takes
- * (Sec. 3.1 phase 1 feeds these outputs to the Sec. 3.2 sums, Delta being the
- * residual A_full - A_loc whose outer products they add up):
- *   delta_hi, delta_lo : bf16 [n_q][num_heads * head_dim], caller-owned, 16-byte
- *                        aligned; Delta = a_full - a_loc of the STORED bf16
- *                        outputs, exact in fp32, written as hi = bf16(Delta)
- *                        and lo = bf16(Delta - hi) (round to nearest even)
- * Every other argument, output and error is that of ispa_attn_dual_ex; on
- * ISPA_ERR_TIMEOUT delta_hi and delta_lo are undefined like the outputs.
- * The pair is formed by the launch that reduces the per-head discrepancy
- * partials (one read of both stored outputs, one write of the pair), so the
- * warmup step's LS call no longer needs a pass of its own over A_loc and A_full.
- */
-ISPA_API ispa_status ispa_attn_dual_delta(const ispa_kv_ring* ring, ispa_window win, const void* q,
-                                 const void* k_cur, const void* v_cur, int32_t n_q, float scale,
-                                 uint32_t flags, void* a_full, void* a_loc, void* delta_hi,
-                                 void* delta_lo, float* disc, float* disc_sq_sum, float* lse_full,
-                                 float* lse_loc, void* workspace, size_t ws_bytes,
-                                 ispa_stream stream);
-
 /* Largest num_heads * n_q that ispa_attn_dual_static accepts (4 MiB of fp32). */
 #define ISPA_DUAL_STATIC_MAX_PARTIALS (1u << 20)
 
@@ -484,28 +462,31 @@ ISPA_API size_t ispa_ls_accumulate_workspace_size(int32_t dim, int64_t T);
  * Add T tokens to the normal-equation sums (Sec. 3.2, "summing the outer
  * products ... during the standard forward pass"):
  *   G += A_loc^T A_loc,  X += A_loc^T Delta,  S += Delta^T Delta,  n += T,
- * Delta = A_full - A_loc taken exactly in fp32 and carried as a bf16 hi + lo
- * pair, products on the tensor cores with fp32 accumulation.
+ * Delta = A_full - A_loc taken exactly in fp32, products on the tensor cores
+ * with fp32 accumulation.  A_loc and Delta enter as fp16, each multiplied by
+ * the power of two that puts its largest magnitude over the call in
+ * [2^14, 2^15); the factors are undone exactly when the sums are added to the
+ * state.  A_loc's bf16 values convert exactly (down to 2^-29 of its largest
+ * magnitude); Delta is rounded once, to 2^-11 relative, which leaves X and S
+ * within about 1e-4 (Frobenius-relative) of the exact sums on typical inputs
+ * and within 2 x 2^-11 in the worst case; the trace form of eps (Eq. 6) and
+ * dW (Eq. 5) are affected far less, because independent roundings cancel in
+ * them.  ISPA_LS_EXACT_DELTA (ispa_ls_accumulate_ex) carries Delta instead as
+ * a bf16 hi + lo pair (2^-16 relative) at twice the tensor work for X and three
+ * times for S.
  *   a_loc, a_full : bf16 [T][dim], dim a multiple of 128 (else UNSUPPORTED).
+ *   workspace     : >= ispa_ls_accumulate_workspace_size(dim, T) bytes.
  */
 ISPA_API ispa_status ispa_ls_accumulate(ispa_ls_state* state, const void* a_loc, const void* a_full,
                                int64_t T, void* workspace, size_t ws_bytes, ispa_stream stream);
 
-/*
- * ispa_ls_accumulate from Delta already split (Sec. 3.2 sums, as above):
- *   a_loc              : bf16 [T][dim]
- *   delta_hi, delta_lo : bf16 [T][dim], Delta = delta_hi + delta_lo (the pair
- *                        ispa_attn_dual_delta writes; any split with
- *                        |lo| <= 2^-8 |hi| gives the same sums to fp32 rounding)
- * No workspace.  Given the pair ispa_attn_dual_delta wrote for a_loc and
- * a_full, the call runs the same products as ispa_ls_accumulate on
- * (a_loc, a_full); the two states differ only in the order in which the fp32
- * partial sums of a tile shared by several CTAs are added.  All pointers
- * 16-byte aligned; dim a multiple of 128 (else UNSUPPORTED).
- */
-ISPA_API ispa_status ispa_ls_accumulate_delta(ispa_ls_state* state, const void* a_loc,
-                                     const void* delta_hi, const void* delta_lo, int64_t T,
-                                     ispa_stream stream);
+/* Option bits of ispa_ls_accumulate_ex. */
+#define ISPA_LS_EXACT_DELTA 1u
+
+/* ispa_ls_accumulate with option bits (unknown bits: ISPA_ERR_INVALID_ARG). */
+ISPA_API ispa_status ispa_ls_accumulate_ex(ispa_ls_state* state, const void* a_loc, const void* a_full,
+                                  int64_t T, uint32_t flags, void* workspace, size_t ws_bytes,
+                                  ispa_stream stream);
 
 /* Workspace bytes of ispa_ls_solve. */
 ISPA_API size_t ispa_ls_solve_workspace_size(int32_t dim, int32_t d_out);

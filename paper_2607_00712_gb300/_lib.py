@@ -25,6 +25,7 @@ ISPA_ERR_TIMEOUT = 5
 ISPA_ERR_CUDA = 6
 ISPA_ERR_WORKSPACE = 7
 ISPA_ATTN_FRAME_CAUSAL = 1   # option bit of the *_ex attention entry points
+ISPA_LS_EXACT_DELTA = 1      # option bit of ispa_ls_accumulate_ex
 ISPA_KV_BF16 = 0             # ring k_format values
 ISPA_KV_K_E4M3 = 1
 ISPA_KV_KV_E4M3 = 2
@@ -96,9 +97,6 @@ _SIGS = {
     "ispa_attn_dual_ex": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                     c_uint32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                     c_void_p, c_size_t, c_void_p]),
-    "ispa_attn_dual_delta": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
-                                       c_uint32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
-                                       c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "ispa_attn_dual_workspace_size": (c_size_t, [c_int32, c_int32]),
     "ispa_attn_dual": (c_int32, [POINTER(KVRing), Window, c_void_p, c_void_p, c_void_p, c_int32, c_float,
                                  c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -118,7 +116,8 @@ _SIGS = {
     "ispa_ls_accumulate_workspace_size": (c_size_t, [c_int32, c_int64]),
     "ispa_ls_accumulate": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
                                      c_void_p]),
-    "ispa_ls_accumulate_delta": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_void_p, c_int64, c_void_p]),
+    "ispa_ls_accumulate_ex": (c_int32, [POINTER(LSState), c_void_p, c_void_p, c_int64, c_uint32, c_void_p,
+                                        c_size_t, c_void_p]),
     "ispa_ls_solve_workspace_size": (c_size_t, [c_int32, c_int32]),
     "ispa_quantize_heads_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "ispa_quantize_q_e4m3": (c_int32, [c_void_p, c_int64, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
@@ -291,15 +290,6 @@ def ispa_attn_dual_ex(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scal
            "ispa_attn_dual_ex")
 
 
-def ispa_attn_dual_delta(ring: KVRing, win: Window, q, k_cur, v_cur, n_q: int, scale: float, flags: int, a_full,
-                         a_loc, delta_hi, delta_lo, disc, disc_sq_sum, lse_full=None, lse_loc=None, workspace=None,
-                         ws_bytes: int = 0, stream=None) -> None:
-    _check(lib().ispa_attn_dual_delta(ctypes.byref(ring), win, _ptr(q), _ptr(k_cur), _ptr(v_cur), n_q, scale,
-                                      flags, _ptr(a_full), _ptr(a_loc), _ptr(delta_hi), _ptr(delta_lo), _ptr(disc),
-                                      _ptr(disc_sq_sum), _ptr(lse_full), _ptr(lse_loc), _ptr(workspace), ws_bytes,
-                                      _stream(stream)), "ispa_attn_dual_delta")
-
-
 def ispa_attn_dual_workspace_size(num_heads: int, n_q: int) -> int:
     return lib().ispa_attn_dual_workspace_size(num_heads, n_q)
 
@@ -374,9 +364,10 @@ def ispa_ls_accumulate(state: LSState, a_loc, a_full, T: int, workspace, ws_byte
                                     ws_bytes, _stream(stream)), "ispa_ls_accumulate")
 
 
-def ispa_ls_accumulate_delta(state: LSState, a_loc, delta_hi, delta_lo, T: int, stream=None) -> None:
-    _check(lib().ispa_ls_accumulate_delta(ctypes.byref(state), _ptr(a_loc), _ptr(delta_hi), _ptr(delta_lo), T,
-                                          _stream(stream)), "ispa_ls_accumulate_delta")
+def ispa_ls_accumulate_ex(state: LSState, a_loc, a_full, T: int, flags: int, workspace, ws_bytes: int,
+                          stream=None) -> None:
+    _check(lib().ispa_ls_accumulate_ex(ctypes.byref(state), _ptr(a_loc), _ptr(a_full), T, flags, _ptr(workspace),
+                                       ws_bytes, _stream(stream)), "ispa_ls_accumulate_ex")
 
 
 def ispa_ls_solve_workspace_size(dim: int, d_out: int) -> int:

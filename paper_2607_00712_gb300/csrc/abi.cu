@@ -706,27 +706,6 @@ ispa_status ispa_attn_dual(const ispa_kv_ring* ring, ispa_window win, const void
                            lse_full, lse_loc, workspace, ws_bytes, stream);
 }
 
-ispa_status ispa_attn_dual_delta(const ispa_kv_ring* ring, ispa_window win, const void* q,
-                                 const void* k_cur, const void* v_cur, int32_t n_q, float scale, uint32_t flags,
-                                 void* a_full, void* a_loc, void* delta_hi, void* delta_lo, float* disc,
-                                 float* disc_sq_sum, float* lse_full, float* lse_loc, void* workspace,
-                                 size_t ws_bytes, ispa_stream stream) {
-  if (!ring || !disc || !disc_sq_sum || !aligned16(delta_hi) || !aligned16(delta_lo) || !aligned16(a_full) ||
-      !aligned16(a_loc))
-    return ISPA_ERR_INVALID_ARG;
-  const size_t need = ispa_attn_dual_workspace_size(ring->num_heads, n_q);
-  if (need == 0) return ISPA_ERR_INVALID_ARG;
-  if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
-  float* part = static_cast<float*>(workspace);
-  const ispa_status st = attn_common(MODE_DUAL, ring, win, q, k_cur, v_cur, n_q, scale, flags, a_full, a_loc,
-                                     lse_full, lse_loc, part, stream);
-  if (st != ISPA_OK) return st;
-  if (launch_disc_split(part, ring->num_heads, n_q, disc, disc_sq_sum, a_loc, a_full, delta_hi, delta_lo,
-                        ring->num_heads * ring->head_dim, stream) != cudaSuccess)
-    return ISPA_ERR_CUDA;
-  return ISPA_OK;
-}
-
 size_t ispa_ls_state_bytes(int32_t dim) {
   if (dim <= 0) return 0;
   return 4ull * dim * dim * sizeof(float);
@@ -745,36 +724,27 @@ size_t ispa_ls_accumulate_workspace_size(int32_t dim, int64_t T) {
   return ls_accumulate_ws_bytes(dim, T);
 }
 
-ispa_status ispa_ls_accumulate(ispa_ls_state* st, const void* a_loc, const void* a_full, int64_t T,
-                               void* workspace, size_t ws_bytes, ispa_stream stream) {
+ispa_status ispa_ls_accumulate_ex(ispa_ls_state* st, const void* a_loc, const void* a_full, int64_t T,
+                                  uint32_t flags, void* workspace, size_t ws_bytes, ispa_stream stream) {
   if (!st || st->dim <= 0 || T <= 0 || T > INT32_MAX || !aligned16(st->gram) || !aligned16(a_loc) ||
       !aligned16(a_full))
     return ISPA_ERR_INVALID_ARG;
+  if (flags & ~static_cast<uint32_t>(ISPA_LS_EXACT_DELTA)) return ISPA_ERR_INVALID_ARG;
   if (st->dim % 128 != 0) return ISPA_ERR_UNSUPPORTED;
   const size_t need = ls_accumulate_ws_bytes(st->dim, T);
   if (!workspace || ws_bytes < need || !aligned16(workspace)) return ISPA_ERR_WORKSPACE;
   int* status = device_status_ptr();
   if (!status) return ISPA_ERR_CUDA;
-  if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, st->gram, status, g_wait_limit.load(),
-                           next_heartbeat_slot(2), stream) != cudaSuccess)
+  if (launch_ls_accumulate(st->dim, T, a_loc, a_full, workspace, (flags & ISPA_LS_EXACT_DELTA) != 0, st->gram,
+                           status, g_wait_limit.load(), next_heartbeat_slot(2), stream) != cudaSuccess)
     return ISPA_ERR_CUDA;
   st->n_tokens += T;
   return ISPA_OK;
 }
 
-ispa_status ispa_ls_accumulate_delta(ispa_ls_state* st, const void* a_loc, const void* delta_hi,
-                                     const void* delta_lo, int64_t T, ispa_stream stream) {
-  if (!st || st->dim <= 0 || T <= 0 || T > INT32_MAX || !aligned16(st->gram) || !aligned16(a_loc) ||
-      !aligned16(delta_hi) || !aligned16(delta_lo))
-    return ISPA_ERR_INVALID_ARG;
-  if (st->dim % 128 != 0) return ISPA_ERR_UNSUPPORTED;
-  int* status = device_status_ptr();
-  if (!status) return ISPA_ERR_CUDA;
-  if (launch_ls_gram(st->dim, T, a_loc, delta_hi, delta_lo, st->gram, status, g_wait_limit.load(),
-                     next_heartbeat_slot(2), stream) != cudaSuccess)
-    return ISPA_ERR_CUDA;
-  st->n_tokens += T;
-  return ISPA_OK;
+ispa_status ispa_ls_accumulate(ispa_ls_state* st, const void* a_loc, const void* a_full, int64_t T,
+                               void* workspace, size_t ws_bytes, ispa_stream stream) {
+  return ispa_ls_accumulate_ex(st, a_loc, a_full, T, 0u, workspace, ws_bytes, stream);
 }
 
 size_t ispa_ls_solve_workspace_size(int32_t dim, int32_t d_out) {

@@ -2,24 +2,27 @@
 //   G += A_loc^T A_loc,  X += A_loc^T Delta,  S += Delta^T Delta,
 // with Delta = A_full - A_loc, on the tensor cores (tcgen05, fp32 in TMEM).
 //
-// Step 1 (split_kernel, HBM-bound): Delta is formed exactly in fp32 from the
-// two bf16 inputs and stored as a bf16 pair hi = bf16(Delta),
-// lo = bf16(Delta - hi), so hi + lo carries Delta to ~2^-16 relative.
-// Step 2: every output tile of the upper blocks is a contraction over tokens, the
-// token axis being the UMMA K dimension:
-//   G tile: a^T a;   X tile: a^T hi + a^T lo;   S tile: hi^T hi + hi^T lo + lo^T hi
-// (the lo^T lo term is below fp32 resolution and dropped).  Both operands
-// are token-major [T][D] in HBM, i.e. MN-major for the UMMA, staged by TMA with
-// 128-byte swizzle, 64 tokens per pipeline stage, one request per operand.
-// Sums reach the fp32 state through vector atomics (flush_block32).
+// Two forms of the operands, both with Delta formed exactly in fp32 from the two bf16 inputs:
+//  * scaled (default): amax_kernel takes max |A_loc| and max |Delta| over the call, and
+//    convert_kernel writes both as fp16 times a power of two that puts the largest
+//    magnitude in [2^14, 2^15) (A_loc's bf16 values convert exactly; Delta rounds once, to
+//    2^-11 relative).  One pass per tile: G = a^T a, X = a^T d, S = d^T d on f16 UMMAs,
+//    each sum multiplied back by its exact power of two before it reaches the state.
+//  * exact (ISPA_LS_EXACT_DELTA): split_kernel stores Delta as the bf16 pair hi = bf16(Delta),
+//    lo = bf16(Delta - hi), ~2^-16 relative; G tile: a^T a, X tile: a^T hi + a^T lo, S tile:
+//    hi^T hi + hi^T lo + lo^T hi (lo^T lo is below fp32 resolution and dropped) on bf16 UMMAs.
+// Every output tile of the upper blocks is a contraction over tokens, the token axis being
+// the UMMA K dimension.  Both operands are token-major [T][D] in HBM, i.e. MN-major for the
+// UMMA, staged by TMA with 128-byte swizzle, 64 tokens per pipeline stage, one request per
+// operand.
 //
 // gram_wide_kernel (D % 256 == 0): 256 x 256 tiles, two 128 x 256 accumulators
 // sharing each B operand, full waves of tiles in a blocked order plus a stream-K
 // tail (see the comment above the kernel).
 //
 // gram_kernel (other D, multiples of 128): 128 x 128 tiles, stream-K over one
-// sequence of steps (tile, pass, 64-token block) -- G tiles (1 pass each), X tiles
-// (2), S tiles (3) -- cut into equal contiguous ranges for a persistent grid of one
+// sequence of steps (tile, pass, 64-token block) -- G tiles, X tiles, S tiles with the
+// passes of the form -- cut into equal contiguous ranges for a persistent grid of one
 // CTA per SM.  A CTA's range covers the tail of one tile, some whole tiles and the
 // head of another; each such segment is summed in one of two TMEM accumulators and
 // added into the state by the epilogue warps while the UMMA warp already fills the
@@ -31,6 +34,8 @@
 #include "delta.cuh"
 #include "internal.h"
 #include "pdl.cuh"
+
+#include <cuda_fp16.h>
 #include "ptx.cuh"
 
 namespace ispa {
@@ -56,20 +61,33 @@ struct GCfg {
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static_assert(OFF_T % 16 == 0, "16-byte aligned staging buffers");
   static_assert(STAGE % 1024 == 0 && BOX % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
-  static constexpr uint32_t IDESC = idesc_bf16(GM, BN, true, true);
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators: 256 or 512 columns
 };
 
-// Operand sources of the passes of each block type: 0 = A_loc, 1 = hi, 2 = lo.
+// Operand sources of the passes of each block type.  Exact form: 0 = A_loc, 1 = hi, 2 = lo;
+// scaled form: 0 = A_loc, 1 = Delta (both fp16, scaled).
 struct Pass {
   int8_t a, b;
 };
-__constant__ Pass kPasses[3][3] = {
-    {{0, 0}, {0, 0}, {0, 0}},  // G: one pass
-    {{0, 1}, {0, 2}, {0, 0}},  // X: two passes
-    {{1, 1}, {1, 2}, {2, 1}},  // S: three passes
+__constant__ Pass kPasses[2][3][3] = {
+    {
+        {{0, 0}, {0, 0}, {0, 0}},  // G: one pass
+        {{0, 1}, {0, 2}, {0, 0}},  // X: two passes
+        {{1, 1}, {1, 2}, {2, 1}},  // S: three passes
+    },
+    {
+        {{0, 0}, {0, 0}, {0, 0}},  // G
+        {{0, 1}, {0, 0}, {0, 0}},  // X
+        {{1, 1}, {0, 0}, {0, 0}},  // S
+    },
 };
-__constant__ int kNumPasses[3] = {1, 2, 3};
+constexpr int kPassesExact[3] = {1, 2, 3};
+constexpr int kPassesScaled[3] = {1, 1, 1};
+
+// The bf16 descriptor with the A and B format fields (bits 7-9, 10-12) set to f16 (0).
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool a_mn_major, bool b_mn_major) {
+  return idesc_bf16(M, N, a_mn_major, b_mn_major) & ~((7u << 7) | (7u << 10));
+}
 
 struct GramParams {
   int32_t D;
@@ -78,30 +96,40 @@ struct GramParams {
   int32_t n_upper;    // upper-block tiles of G (and of S)
   int32_t n_full;     // tiles of X
   int32_t total;      // steps over all tiles
+  int32_t form;       // 0 exact (bf16 hi / lo), 1 scaled (fp16)
+  int32_t passes[3];  // passes per tile of G, X, S
+  uint32_t idesc;     // UMMA instruction descriptor of the form
+  const float* unscale;   // scaled form: the factor of G, X, S sums; null: 1
   float* gram;        // [2D][2D]
   int* status;
   uint64_t wait_limit_ns;
   uint32_t* heartbeat;
 };
 
+// Kernel parameters indexed by a run-time kind without a local copy of the arrays.
+__device__ __forceinline__ int32_t pick3(const int32_t (&a)[3], int k) {
+  return k == 0 ? a[0] : (k == 1 ? a[1] : a[2]);
+}
+
 // Step g of the global sequence -> tile (item, numbered as decode_tile expects) and its
-// first step.  Tiles: n_upper G tiles of n_kt steps, n_full X tiles of 2 n_kt, n_upper S
-// tiles of 3 n_kt.
+// first step.  Tiles: n_upper G tiles, n_full X tiles, n_upper S tiles, each of
+// passes[kind] * n_kt steps.
 __device__ __forceinline__ void step_item(const GramParams& p, int g, int& item, int& first) {
   const int n_kt = p.n_ktiles;
-  const int g_end = p.n_upper * n_kt;
-  const int x_end = g_end + p.n_full * 2 * n_kt;
+  const int lg = p.passes[0] * n_kt, lx = p.passes[1] * n_kt, ls = p.passes[2] * n_kt;
+  const int g_end = p.n_upper * lg;
+  const int x_end = g_end + p.n_full * lx;
   if (g < g_end) {
-    item = g / n_kt;
-    first = item * n_kt;
+    item = g / lg;
+    first = item * lg;
   } else if (g < x_end) {
-    const int i = (g - g_end) / (2 * n_kt);
+    const int i = (g - g_end) / lx;
     item = p.n_upper + i;
-    first = g_end + i * 2 * n_kt;
+    first = g_end + i * lx;
   } else {
-    const int i = (g - x_end) / (3 * n_kt);
+    const int i = (g - x_end) / ls;
     item = p.n_upper + p.n_full + i;
-    first = x_end + i * 3 * n_kt;
+    first = x_end + i * ls;
   }
 }
 
@@ -145,14 +173,16 @@ __device__ __forceinline__ void decode_tile(int item, int D, int& kind, int& bi,
 // q ^ (t & 7): no bank conflicts on the write or the read) so that each atomic
 // instruction of the warp covers 4 rows x 128 contiguous bytes instead of 32 rows x
 // 16 bytes; measured on GB300 this made the whole accumulate 23-36 % faster.
-__device__ __forceinline__ void flush_block32(uint32_t taddr, float4* tbuf, float* dst, size_t ld, int lane) {
+__device__ __forceinline__ void flush_block32(uint32_t taddr, float4* tbuf, float* dst, size_t ld, int lane,
+                                              float scale) {
   uint32_t v[32];
   tmem_ld32(taddr, v);
   tmem_wait_ld32(v);
 #pragma unroll
   for (int q = 0; q < 8; ++q)
-    tbuf[lane * 8 + (q ^ (lane & 7))] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                                    __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+    tbuf[lane * 8 + (q ^ (lane & 7))] =
+        make_float4(__uint_as_float(v[4 * q]) * scale, __uint_as_float(v[4 * q + 1]) * scale,
+                    __uint_as_float(v[4 * q + 2]) * scale, __uint_as_float(v[4 * q + 3]) * scale);
   __syncwarp();
   const int rr = lane >> 3, qq = lane & 7;
 #pragma unroll
@@ -172,6 +202,99 @@ __global__ void __launch_bounds__(256) split_kernel(const uint4* __restrict__ a_
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride)
     split_delta8(a_loc[i], a_full[i], hi[i], lo[i]);
+}
+
+// Largest |value| of a block's 256 threads (all threads call it; the result is in every thread).
+__device__ __forceinline__ float block_max256(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  __syncthreads();   // red may still be read by a previous call
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  v = red[0];
+#pragma unroll
+  for (int w = 1; w < 8; ++w) v = fmaxf(v, red[w]);
+  return v;
+}
+
+// Scaled form, pass 1: max |A_loc| and max |Delta| of each block's words -> part[b], part[nb + b].
+__global__ void __launch_bounds__(256) amax_kernel(const uint4* __restrict__ a_loc, const uint4* __restrict__ a_full,
+                                                   int64_t n_words, float* __restrict__ part) {
+  pdl_trigger();   // convert_kernel may set itself up meanwhile
+  __shared__ float red[8];
+  float ma = 0.f, md = 0.f;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
+    const uint4 a = a_loc[i], f = a_full[i];
+    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+      const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
+      ma = fmaxf(ma, fmaxf(fabsf(a0), fabsf(a1)));
+      md = fmaxf(md, fmaxf(fabsf(f0 - a0), fabsf(f1 - a1)));
+    }
+  }
+  ma = block_max256(ma, red);
+  md = block_max256(md, red);
+  if (threadIdx.x == 0) {
+    part[blockIdx.x] = ma;
+    part[gridDim.x + blockIdx.x] = md;
+  }
+}
+
+// Exponent s with amax * 2^s in [2^14, 2^15) (0 for amax = 0), kept in [-60, 60] so that
+// 2^s and 2^-2s are normal fp32 numbers.
+__device__ __forceinline__ int scale_exp(float amax) {
+  if (!(amax > 0.f)) return 0;
+  const int e = static_cast<int>((__float_as_uint(amax) >> 23) & 0xFF) - 127;
+  return max(-60, min(60, 14 - e));
+}
+__device__ __forceinline__ float pow2f(int s) { return __uint_as_float(static_cast<uint32_t>(127 + s) << 23); }
+
+// Scaled form, pass 2: the call's maxima from amax_kernel's nb partials, then
+// a16 = fp16(A_loc * 2^sa) (exact) and d16 = fp16(Delta * 2^sd) (one rounding), eight
+// features per thread and step; block 0 stores the factors 2^-2sa, 2^-(sa+sd), 2^-2sd that
+// take the G, X and S sums back to the inputs' scale.
+__global__ void __launch_bounds__(256) convert_kernel(const uint4* __restrict__ a_loc,
+                                                      const uint4* __restrict__ a_full, int64_t n_words,
+                                                      const float* __restrict__ part, int nb,
+                                                      uint4* __restrict__ a16, uint4* __restrict__ d16,
+                                                      float* __restrict__ unscale) {
+  pdl_wait();   // amax_kernel's partials
+  __shared__ float red[8];
+  float ma = 0.f, md = 0.f;
+  for (int b = threadIdx.x; b < nb; b += blockDim.x) {
+    ma = fmaxf(ma, part[b]);
+    md = fmaxf(md, part[nb + b]);
+  }
+  ma = block_max256(ma, red);
+  md = block_max256(md, red);
+  const int sa = scale_exp(ma), sd = scale_exp(md);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    unscale[0] = pow2f(-2 * sa);
+    unscale[1] = pow2f(-(sa + sd));
+    unscale[2] = pow2f(-2 * sd);
+  }
+  pdl_trigger();   // the Gram kernel may set itself up meanwhile
+  const float ka = pow2f(sa), kd = pow2f(sd);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
+    const uint4 a = a_loc[i], f = a_full[i];
+    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
+    uint32_t ow[4], dw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+      const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
+      __half2 h = __floats2half2_rn(a0 * ka, a1 * ka);
+      ow[e] = *reinterpret_cast<uint32_t*>(&h);
+      h = __floats2half2_rn((f0 - a0) * kd, (f1 - a1) * kd);
+      dw[e] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    a16[i] = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+    d16[i] = make_uint4(dw[0], dw[1], dw[2], dw[3]);
+  }
 }
 
 template <int BN>
@@ -236,7 +359,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
       int item = -1, first = 0, kind = 0, bi = 0, bj = 0;
       for (int g = g0; g < g1; ++g) {
         const int i = g - g0;
-        if (item < 0 || g >= first + kNumPasses[kind] * n_kt) {
+        if (item < 0 || g >= first + pick3(p.passes, kind) * n_kt) {
           step_item(p, g, item, first);
           decode_tile<BN>(item, p.D, kind, bi, bj);
         }
@@ -247,8 +370,8 @@ __global__ void __launch_bounds__(G_THREADS, 1)
         if (!mbar_wait(empty0 + 8 * st, ((i / GST) & 1) ^ 1, wc, 21, i)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, C::STAGE);
         const uint32_t sa = sbase + st * C::STAGE, sb = sa + C::A_BYTES;
-        const CUtensorMap* ma = map_r(kPasses[kind][pass].a);
-        const CUtensorMap* mb = map_c(kPasses[kind][pass].b);
+        const CUtensorMap* ma = map_r(kPasses[p.form][kind][pass].a);
+        const CUtensorMap* mb = map_c(kPasses[p.form][kind][pass].b);
         // one request per operand: (64 features, GK tokens, GM/64 or BN/64 feature blocks)
         tma_load_3d(sa, ma, full0 + 8 * st, 0, tok, bi * (GM / 64));
         tma_load_3d(sb, mb, full0 + 8 * st, 0, tok, bj * (BN / 64));
@@ -270,7 +393,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
           step_item(p, g, item, first);
           int kind, bi, bj;
           decode_tile<BN>(item, p.D, kind, bi, bj);
-          last = first + kNumPasses[kind] * n_kt;
+          last = first + pick3(p.passes, kind) * n_kt;
           const int b = seg & 1;
           if (!mbar_wait(acce0 + 8 * b, ((seg >> 1) & 1) ^ 1, wc, 24, seg)) {
             ok = false;
@@ -289,7 +412,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
         const bool seg_first = (g == g0) || (g == first);
 #pragma unroll
         for (int k = 0; k < GK / 16; ++k)
-          umma_ss(acc, sw128_desc(sa + k * 2048, C::BOX, 1024), sw128_desc(sb + k * 2048, C::BOX, 1024), C::IDESC,
+          umma_ss(acc, sw128_desc(sa + k * 2048, C::BOX, 1024), sw128_desc(sb + k * 2048, C::BOX, 1024), p.idesc,
                   (!seg_first || k > 0) ? 1u : 0u);
         tc_commit(empty0 + 8 * st);
         if (g + 1 == g1 || g + 1 == last) tc_commit(accf0 + 8 * (seg & 1));
@@ -319,9 +442,10 @@ __global__ void __launch_bounds__(G_THREADS, 1)
       const int row0 = (kind == 2 ? D : 0) + bi * GM;
       const int col0 = (kind == 0 ? 0 : D) + bj * BN;
       float* gblk = p.gram + static_cast<size_t>(row0 + quarter * 32) * (2 * D) + col0;
+      const float scale = p.unscale ? p.unscale[kind] : 1.f;
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c)
-        flush_block32(lane_base + b * BN + 32 * c, tbuf, gblk + 32 * c, 2 * static_cast<size_t>(D), lane);
+        flush_block32(lane_base + b * BN + 32 * c, tbuf, gblk + 32 * c, 2 * static_cast<size_t>(D), lane, scale);
       tc_fence_before();
       mbar_arrive(acce0 + 8 * b);   // accumulator b may be overwritten
     }
@@ -364,7 +488,6 @@ constexpr int W_N_BAR = 2 * W_ST + 1 + 2 + 1;   // full/empty stages, acc full, 
 constexpr int W_OFF_T = (W_OFF_BAR + W_N_BAR * 8 + 16 + 1023) / 1024 * 1024;   // epilogue staging, 8 warps x 4 KB
 constexpr int W_SMEM = W_OFF_T + 8 * 32 * 32 * 4;
 constexpr int W_BAND = 8;               // tile columns per band of the blocked order
-constexpr uint32_t W_IDESC = idesc_bf16(128, 256, true, true);
 static_assert(W_SMEM <= 232448, "shared memory per CTA");
 static_assert(W_OFF_T % 1024 == 0, "staging blocks on the 1 KB period of the 128-byte swizzle");
 static_assert(W_STAGE % 1024 == 0, "swizzle atoms need 1 KB aligned boxes");
@@ -376,6 +499,10 @@ struct WideParams {
   int32_t U[3];        // tiles per kind: G (upper, diagonal included), X (all), S (upper)
   int32_t waves[3];    // full waves per kind
   int64_t tail_total;  // steps of the shared tail
+  int32_t form;        // 0 exact (bf16 hi / lo), 1 scaled (fp16)
+  int32_t passes[3];   // passes per tile of G, X, S
+  uint32_t idesc;      // UMMA instruction descriptor of the form
+  const float* unscale;   // scaled form: the factor of G, X, S sums; null: 1
   float* gram;
   int* status;
   uint64_t wait_limit_ns;
@@ -399,11 +526,6 @@ __device__ __forceinline__ void wide_tile(int kind, int t, int NB, int& bi, int&
     }
   }
   bi = bj = 0;
-}
-
-// Kernel parameters indexed by a run-time kind without a local copy of the arrays.
-__device__ __forceinline__ int32_t pick3(const int32_t (&a)[3], int k) {
-  return k == 0 ? a[0] : (k == 1 ? a[1] : a[2]);
 }
 
 struct WSeg {
@@ -431,7 +553,7 @@ __device__ __forceinline__ bool wit_next(const WideParams& p, WIter& it, WSeg& s
       s.kind = it.k;
       wide_tile(it.k, it.w * G + static_cast<int>(blockIdx.x), p.NB, s.bi, s.bj);
       s.s0 = 0;
-      s.s1 = kNumPasses[it.k] * p.n_ktiles;
+      s.s1 = pick3(p.passes, it.k) * p.n_ktiles;
       ++it.w;
       return true;
     }
@@ -442,12 +564,12 @@ __device__ __forceinline__ bool wit_next(const WideParams& p, WIter& it, WSeg& s
   int64_t g = it.g;
   int k = 0;
   for (; k < 3; ++k) {
-    const int64_t n = static_cast<int64_t>(pick3(p.U, k) - pick3(p.waves, k) * G) * kNumPasses[k] * p.n_ktiles;
+    const int64_t n = static_cast<int64_t>(pick3(p.U, k) - pick3(p.waves, k) * G) * pick3(p.passes, k) * p.n_ktiles;
     if (g < n) break;
     g -= n;
   }
   if (k >= 3) return false;
-  const int64_t L = static_cast<int64_t>(kNumPasses[k]) * p.n_ktiles;
+  const int64_t L = static_cast<int64_t>(pick3(p.passes, k)) * p.n_ktiles;
   s.kind = k;
   wide_tile(k, pick3(p.waves, k) * G + static_cast<int>(g / L), p.NB, s.bi, s.bj);
   s.s0 = static_cast<int>(g % L);
@@ -524,8 +646,8 @@ __global__ void __launch_bounds__(W_THREADS, 1)
           mbar_arrive_expect_tx(full0 + 8 * sl, W_STAGE);
           const uint32_t sa = sbase + sl * W_STAGE, sb = sa + W_OPER;
           // one request per operand: (64 features, GK tokens, 4 feature blocks)
-          tma_load_3d(sa, map(kPasses[sg.kind][pass].a), full0 + 8 * sl, 0, tok, sg.bi * 4);
-          tma_load_3d(sb, map(kPasses[sg.kind][pass].b), full0 + 8 * sl, 0, tok, sg.bj * 4);
+          tma_load_3d(sa, map(kPasses[p.form][sg.kind][pass].a), full0 + 8 * sl, 0, tok, sg.bi * 4);
+          tma_load_3d(sb, map(kPasses[p.form][sg.kind][pass].b), full0 + 8 * sl, 0, tok, sg.bj * 4);
         }
       }
       for (int k = i > W_ST ? i - W_ST : 0; k < i; ++k)
@@ -556,8 +678,8 @@ __global__ void __launch_bounds__(W_THREADS, 1)
           for (int k = 0; k < GK / 16; ++k) {
             const uint32_t acc = (st != sg.s0 || k > 0) ? 1u : 0u;
             const uint64_t db = sw128_desc(sb + k * 2048, W_BOX, 1024);
-            umma_ss(tmem, sw128_desc(sa + k * 2048, W_BOX, 1024), db, W_IDESC, acc);
-            umma_ss(tmem + 256, sw128_desc(sa + 2 * W_BOX + k * 2048, W_BOX, 1024), db, W_IDESC, acc);
+            umma_ss(tmem, sw128_desc(sa + k * 2048, W_BOX, 1024), db, p.idesc, acc);
+            umma_ss(tmem + 256, sw128_desc(sa + 2 * W_BOX + k * 2048, W_BOX, 1024), db, p.idesc, acc);
           }
           tc_commit(empty0 + 8 * sl);
         }
@@ -593,6 +715,7 @@ __global__ void __launch_bounds__(W_THREADS, 1)
       tc_fence_after();
       const int row0 = (sg.kind == 2 ? D : 0) + sg.bi * 256 + half * 128 + quarter * 32;
       const int col0 = (sg.kind == 0 ? 0 : D) + sg.bj * 256;
+      const float scale = p.unscale ? p.unscale[sg.kind] : 1.f;
 #pragma unroll 1
       for (int c = 0; c < 256 / 32; ++c) {
         uint32_t v[32];
@@ -606,8 +729,9 @@ __global__ void __launch_bounds__(W_THREADS, 1)
         __syncwarp();
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-          tbuf[lane * 8 + (q ^ (lane & 7))] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                                          __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+          tbuf[lane * 8 + (q ^ (lane & 7))] =
+              make_float4(__uint_as_float(v[4 * q]) * scale, __uint_as_float(v[4 * q + 1]) * scale,
+                          __uint_as_float(v[4 * q + 2]) * scale, __uint_as_float(v[4 * q + 3]) * scale);
         fence_proxy_async_smem();   // these generic-proxy writes before the bulk copy reads them
         __syncwarp();
         if (lane == 0) {
@@ -630,9 +754,9 @@ __global__ void __launch_bounds__(W_THREADS, 1)
   }
 }
 
-static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
-                                    float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
-                                    cudaStream_t s) {
+static cudaError_t launch_gram_wide(int32_t D, int64_t T, int form, const void* op0, const void* op1,
+                                    const void* op2, const float* unscale, float* gram, int* status,
+                                    uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -642,8 +766,10 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   }
   // [T][D] operands viewed as (64 features, T tokens, D/64 feature blocks); one box
   // (64, GK, 4) is a 256-feature slice of GK tokens as 4 swizzled [GK][128 B] blocks
+  // (the maps' bf16 element type only sets the 2-byte element size and the zero fill: the
+  // scaled form's fp16 operands go through the same maps)
   CUtensorMap tm[3], tm_state;
-  const void* srcs[3] = {a_loc, hi, lo};
+  const void* srcs[3] = {op0, op1, op2};
   for (int i = 0; i < 3; ++i)
     if (!encode_tmap_3d(&tm[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, 4))
       return cudaErrorInvalidValue;
@@ -659,7 +785,11 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   p.U[0] = n_upper;
   p.U[1] = p.NB * p.NB;
   p.U[2] = n_upper;
-  const int passes[3] = {1, 2, 3};
+  const int* passes = form ? kPassesScaled : kPassesExact;
+  p.form = form;
+  for (int k = 0; k < 3; ++k) p.passes[k] = passes[k];
+  p.idesc = form ? idesc_f16(128, 256, true, true) : idesc_bf16(128, 256, true, true);
+  p.unscale = unscale;
   int64_t total = 0;
   for (int k = 0; k < 3; ++k) total += static_cast<int64_t>(p.U[k]) * passes[k] * p.n_ktiles;
   if (total > INT32_MAX) return cudaErrorInvalidValue;
@@ -678,15 +808,21 @@ static cudaError_t launch_gram_wide(int32_t D, int64_t T, const void* a_loc, con
   return launch_pdl(gram_wide_kernel, grid, dim3(W_THREADS), W_SMEM, s, tm[0], tm[1], tm[2], tm_state, p);
 }
 
-size_t ls_accumulate_ws_bytes(int32_t D, int64_t T) {
-  // hi and lo, each bf16 [T][D], 256-byte aligned
-  const size_t one = (static_cast<size_t>(T) * D * 2 + 255) & ~static_cast<size_t>(255);
-  return 2 * one;
+// The workspace of one call: two 2-byte [T][D] operands (hi and lo, or the scaled A_loc and
+// Delta), 256-byte aligned, then the scaled form's block maxima and its three factors.
+constexpr int kAmaxBlocks = 1024;   // at most this many amax_kernel blocks
+constexpr size_t kAmaxBytes = (2 * kAmaxBlocks + 4) * sizeof(float);
+
+static size_t ls_operand_bytes(int32_t D, int64_t T) {
+  return (static_cast<size_t>(T) * D * 2 + 255) & ~static_cast<size_t>(255);
 }
 
+size_t ls_accumulate_ws_bytes(int32_t D, int64_t T) { return 2 * ls_operand_bytes(D, T) + kAmaxBytes; }
+
 template <int BN>
-static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo,
-                               float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
+static cudaError_t launch_gram(int32_t D, int64_t T, int form, const void* op0, const void* op1, const void* op2,
+                               const float* unscale, float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
+                               cudaStream_t s) {
   using C = GCfg<BN>;
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
@@ -701,7 +837,7 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   // (measured on GB300: 11 % faster than one 2-D request per 64-feature block at hidden
   // 1536, 1 % at hidden 5120)
   CUtensorMap tr[3], tc[3];
-  const void* srcs[3] = {a_loc, hi, lo};
+  const void* srcs[3] = {op0, op1, op2};
   for (int i = 0; i < 3; ++i)
     if (!encode_tmap_3d(&tr[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, GM / 64) ||
         !encode_tmap_3d(&tc[i], srcs[i], 64, T, D / 64, static_cast<uint64_t>(D) * 2, 128, 64, GK, BN / 64))
@@ -715,7 +851,13 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
   p.n_ktiles = static_cast<int32_t>((T + GK - 1) / GK);
   p.n_upper = n_upper;
   p.n_full = RB * CB;
-  const int64_t total = static_cast<int64_t>(p.n_ktiles) * (n_upper * 1 + p.n_full * 2 + n_upper * 3);
+  const int* passes = form ? kPassesScaled : kPassesExact;
+  p.form = form;
+  for (int k = 0; k < 3; ++k) p.passes[k] = passes[k];
+  p.idesc = form ? idesc_f16(GM, BN, true, true) : idesc_bf16(GM, BN, true, true);
+  p.unscale = unscale;
+  const int64_t total =
+      static_cast<int64_t>(p.n_ktiles) * (n_upper * passes[0] + p.n_full * passes[1] + n_upper * passes[2]);
   if (total > INT32_MAX) return cudaErrorInvalidValue;
   p.total = static_cast<int32_t>(total);
   p.gram = gram;
@@ -730,29 +872,42 @@ static cudaError_t launch_gram(int32_t D, int64_t T, const void* a_loc, const vo
 }
 
 cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full, void* ws,
-                                 float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
+                                 bool exact, float* gram, int* status, uint64_t wait_limit_ns, uint32_t* hb,
                                  cudaStream_t s) {
-  const size_t one = ls_accumulate_ws_bytes(D, T) / 2;
-  uint8_t* hi = static_cast<uint8_t*>(ws);
-  uint8_t* lo = hi + one;
+  const size_t one = ls_operand_bytes(D, T);
+  uint8_t* op1 = static_cast<uint8_t*>(ws);
+  uint8_t* op2 = op1 + one;
+  float* part = reinterpret_cast<float*>(op2 + one);
+  float* unscale = part + 2 * kAmaxBlocks;
   const int64_t n_words = static_cast<int64_t>(T) * D / 8;
   int dev = 0, sms = 152;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int64_t blocks = (n_words + 255) / 256;
   if (blocks > static_cast<int64_t>(sms) * 8) blocks = static_cast<int64_t>(sms) * 8;
-  split_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
-      static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), reinterpret_cast<uint4*>(hi),
-      reinterpret_cast<uint4*>(lo), n_words);
+  if (exact) {
+    // hi, lo of Delta; the Gram kernel reads A_loc itself
+    split_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+        static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), reinterpret_cast<uint4*>(op1),
+        reinterpret_cast<uint4*>(op2), n_words);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    if (D % 256 == 0) return launch_gram_wide(D, T, 0, a_loc, op1, op2, nullptr, gram, status, wait_limit_ns, hb, s);
+    return launch_gram<128>(D, T, 0, a_loc, op1, op2, nullptr, gram, status, wait_limit_ns, hb, s);
+  }
+  // scaled A_loc (op1) and Delta (op2) in fp16
+  int nb = static_cast<int>(blocks < kAmaxBlocks ? blocks : kAmaxBlocks);
+  amax_kernel<<<static_cast<unsigned>(nb), 256, 0, s>>>(static_cast<const uint4*>(a_loc),
+                                                        static_cast<const uint4*>(a_full), n_words, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  return launch_ls_gram(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
-}
-
-cudaError_t launch_ls_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo, float* gram,
-                           int* status, uint64_t wait_limit_ns, uint32_t* hb, cudaStream_t s) {
-  if (D % 256 == 0) return launch_gram_wide(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
-  return launch_gram<128>(D, T, a_loc, hi, lo, gram, status, wait_limit_ns, hb, s);
+  e = launch_pdl(convert_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s,
+                 static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), n_words,
+                 static_cast<const float*>(part), nb, reinterpret_cast<uint4*>(op1), reinterpret_cast<uint4*>(op2),
+                 unscale);
+  if (e != cudaSuccess) return e;
+  if (D % 256 == 0) return launch_gram_wide(D, T, 1, op1, op2, op2, unscale, gram, status, wait_limit_ns, hb, s);
+  return launch_gram<128>(D, T, 1, op1, op2, op2, unscale, gram, status, wait_limit_ns, hb, s);
 }
 
 }  // namespace ispa

@@ -67,11 +67,6 @@ cudaError_t launch_attention(int head_dim, const CUtensorMap* tm_q, const CUtens
 // disc[t] = sqrt(sum_h part[h][t]); *disc_sq_sum += sum_t sum_h part[h][t]
 cudaError_t launch_disc_reduce(const float* part, int32_t H, int32_t n_q, float* disc,
                                float* disc_sq_sum, cudaStream_t s);
-// The same reduction fused with the split of Delta = a_full - a_loc ([n_q][D] bf16 each)
-// into the bf16 pair hi, lo that launch_ls_gram takes.
-cudaError_t launch_disc_split(const float* part, int32_t H, int32_t n_q, float* disc, float* disc_sq_sum,
-                              const void* a_loc, const void* a_full, void* hi, void* lo, int32_t D,
-                              cudaStream_t s);
 
 // O = 0 and LSE = -inf for an empty key set (the history branch with no history).
 cudaError_t launch_empty_branch(void* out, float* lse, int32_t n_q, int32_t H, int32_t d, cudaStream_t s);
@@ -97,14 +92,12 @@ struct AppendParams {
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 
 // ------------------------------------------------------------ least squares
-// Accumulate the upper blocks of [A | dlt]^T [A | dlt] into the fp32 state.
-cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full,
-                                 void* ws, float* gram, int* status, uint64_t wait_limit_ns,
+// Accumulate the upper blocks of [A | dlt]^T [A | dlt] into the fp32 state; exact: Delta as a
+// bf16 hi / lo pair, else A_loc and Delta as scaled fp16.
+cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const void* a_full, void* ws,
+                                 bool exact, float* gram, int* status, uint64_t wait_limit_ns,
                                  uint32_t* heartbeat, cudaStream_t s);
 size_t ls_accumulate_ws_bytes(int32_t D, int64_t T);
-// The same from Delta already split into its bf16 hi / lo pair ([T][D] each).
-cudaError_t launch_ls_gram(int32_t D, int64_t T, const void* a_loc, const void* hi, const void* lo, float* gram,
-                           int* status, uint64_t wait_limit_ns, uint32_t* heartbeat, cudaStream_t s);
 
 size_t ls_solve_ws_bytes(int32_t D, int32_t d_out);
 // Returns ISPA_OK, ISPA_ERR_NOT_SPD or ISPA_ERR_CUDA; synchronises the stream.

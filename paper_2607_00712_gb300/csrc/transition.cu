@@ -9,9 +9,7 @@
 #include <algorithm>
 #include <vector>
 
-#include "delta.cuh"
 #include "internal.h"
-#include "pdl.cuh"
 
 namespace ispa {
 
@@ -176,61 +174,7 @@ int grid_for(int64_t n, int threads) {
 bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 
-// The dual pass's discrepancy reduction (blocks [0, n_disc_blocks), as disc_reduce_kernel) and,
-// in the remaining blocks, Delta = A_full - A_loc of the stored outputs as its bf16 pair
-// hi = bf16(Delta), lo = bf16(Delta - hi), eight features per thread and step.
-__global__ void __launch_bounds__(256) disc_split_kernel(const float* __restrict__ part, int H, int n_q,
-                                                         float* __restrict__ disc, float* __restrict__ disc_sq_sum,
-                                                         int n_disc_blocks, const uint4* __restrict__ a_loc,
-                                                         const uint4* __restrict__ a_full, uint4* __restrict__ hi,
-                                                         uint4* __restrict__ lo, int64_t n_words) {
-  pdl_trigger();   // the Gram kernel after this one may set itself up meanwhile
-  if (static_cast<int>(blockIdx.x) >= n_disc_blocks) {
-    const int64_t stride = static_cast<int64_t>(gridDim.x - n_disc_blocks) * blockDim.x;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x - n_disc_blocks) * blockDim.x + threadIdx.x; i < n_words;
-         i += stride)
-      split_delta8(a_loc[i], a_full[i], hi[i], lo[i]);
-    return;
-  }
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  float v = 0.f;
-  if (t < n_q) {
-    for (int h = 0; h < H; ++h) v += part[static_cast<size_t>(h) * n_q + t];
-    disc[t] = sqrtf(v);
-  }
-  __shared__ float red[8];
-  float w = v;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = w;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    w = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-    if (threadIdx.x == 0) atomicAdd(disc_sq_sum, w);
-  }
-}
-
 }  // namespace
-
-cudaError_t launch_disc_split(const float* part, int32_t H, int32_t n_q, float* disc, float* disc_sq_sum,
-                              const void* a_loc, const void* a_full, void* hi, void* lo, int32_t D,
-                              cudaStream_t s) {
-  if (n_q <= 0) return cudaSuccess;
-  const int n_disc = (n_q + 255) / 256;
-  const int64_t n_words = static_cast<int64_t>(n_q) * D / 8;
-  int dev = 0, sms = 152;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int64_t blocks = (n_words + 255) / 256;
-  if (blocks > static_cast<int64_t>(sms) * 8) blocks = static_cast<int64_t>(sms) * 8;
-  disc_split_kernel<<<static_cast<unsigned>(n_disc + blocks), 256, 0, s>>>(
-      part, H, n_q, disc, disc_sq_sum, n_disc, static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full),
-      static_cast<uint4*>(hi), static_cast<uint4*>(lo), n_words);
-  return cudaGetLastError();
-}
-
 
 cudaError_t launch_empty_branch(void* out, float* lse, int32_t n_q, int32_t H, int32_t d, cudaStream_t s) {
   const int64_t words = static_cast<int64_t>(n_q) * H * d * 2 / 16;

@@ -156,25 +156,17 @@ def test_attention_option_validation_without_gpu():
                                16, 1 << 20, None) == abi.ISPA_ERR_INVALID_ARG
 
 
-def test_delta_entry_points_validation_without_gpu():
+def test_ls_accumulate_option_validation_without_gpu():
     L = abi.lib()
-    r = KVRing(2, 64, 16, 4, 0, 0, 2, 16, 16)
-    # ring, win, q, k_cur, v_cur, n_q, scale, flags, a_full, a_loc, hi, lo, disc, dsum, lse x2, ws, ws_bytes
-    args = [ctypes.byref(r), Window(0, 1), 16, 16, 16, 32, 0.0, 0, 16, 16, 16, 16, 16, 16, None, None, 16, 1 << 20,
-            None]
-    for i, bad in [(10, None), (11, None), (10, 18), (11, 24)]:   # a missing or misaligned hi / lo
-        a = list(args)
-        a[i] = bad
-        assert L.ispa_attn_dual_delta(*a) == abi.ISPA_ERR_INVALID_ARG, (i, bad)
-    a = list(args)
-    a[16] = None
-    assert L.ispa_attn_dual_delta(*a) == abi.ISPA_ERR_WORKSPACE
-    st = LSState(100, 0, 0, 16)
-    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, 16, 10, None) == abi.ISPA_ERR_UNSUPPORTED
     st = LSState(128, 0, 0, 16)
-    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, 16, 0, None) == abi.ISPA_ERR_INVALID_ARG
-    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 24, 16, 10, None) == abi.ISPA_ERR_INVALID_ARG
-    assert L.ispa_ls_accumulate_delta(ctypes.byref(st), 16, 16, None, 10, None) == abi.ISPA_ERR_INVALID_ARG
+    # an unknown option bit
+    assert L.ispa_ls_accumulate_ex(ctypes.byref(st), 16, 16, 10, 2, 16, 1 << 30, None) == abi.ISPA_ERR_INVALID_ARG
+    # the exact form still needs its workspace; dim not a multiple of 128 is unsupported in both
+    assert L.ispa_ls_accumulate_ex(ctypes.byref(st), 16, 16, 10, abi.ISPA_LS_EXACT_DELTA, None, 0,
+                                   None) == abi.ISPA_ERR_WORKSPACE
+    st = LSState(100, 0, 0, 16)
+    assert L.ispa_ls_accumulate_ex(ctypes.byref(st), 16, 16, 10, abi.ISPA_LS_EXACT_DELTA, 16, 1 << 30,
+                                   None) == abi.ISPA_ERR_UNSUPPORTED
     assert st.n_tokens == 0
 
 

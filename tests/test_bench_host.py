@@ -94,13 +94,18 @@ def test_ls_flops_method_and_tile_work():
     # method work 2T(2D^2 + D): 44.2 GFLOP for the 1.3B step (T 4680, D 1536), 490.8 for 14B
     m, t = bench.ls_flops(1536, 4680)
     assert abs(m / 1e9 - 44.18) < 0.01
-    # 256 x 256 tiles: 6 x 6 grid, 21 upper tiles; 21 (G) + 2 * 36 (X) + 3 * 21 (S) = 156 tile-passes
-    assert t == 156 * 2.0 * 256 * 256 * 4680
+    # 256 x 256 tiles: 6 x 6 grid, 21 upper tiles; scaled form one pass per tile: 21 + 36 + 21 = 78
+    assert t == 78 * 2.0 * 256 * 256 * 4680
+    # exact form: 21 (G) + 2 * 36 (X) + 3 * 21 (S) = 156 tile-passes
+    _, te = bench.ls_flops(1536, 4680, exact=True)
+    assert te == 156 * 2.0 * 256 * 256 * 4680
     m14, _ = bench.ls_flops(5120, 4680)
     assert abs(m14 / 1e9 - 490.8) < 0.1
     # a width with no 256 tiling falls back to 128 x 128 tiles
-    _, t384 = bench.ls_flops(384, 10)
+    _, t384 = bench.ls_flops(384, 10, exact=True)
     assert t384 == (6 + 2 * 9 + 3 * 6) * 2.0 * 128 * 128 * 10
+    _, t384s = bench.ls_flops(384, 10)
+    assert t384s == (6 + 9 + 6) * 2.0 * 128 * 128 * 10
 
 
 def test_modes_rates_and_fractions():

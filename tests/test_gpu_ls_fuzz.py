@@ -1,6 +1,7 @@
 """Seeded fuzz of the LS accumulation (Sec. 3.2, Eq. 5) through the C-ABI.
 
-Random hidden sizes (both Gram kernels: 256 x 256 tiles when the size is a multiple of 256,
+Both operand forms (scaled fp16, the default, and the exact bf16 hi / lo pair), random hidden
+sizes (both Gram kernels: 256 x 256 tiles when the size is a multiple of 256,
 128 x 128 tiles otherwise), random token counts (ragged last 64-token block), one to three
 accumulate calls into the same state, and shapes whose tile counts exceed the grid so that the
 lockstep-wave phase of the wide kernel runs, not only its stream-K tail.  Every maintained
@@ -48,15 +49,17 @@ def _maintained_mask(D):
     return keep
 
 
+@pytest.mark.parametrize("exact", [False, True], ids=["scaled", "exact"])
 @pytest.mark.parametrize("D,Ts", _cases(), ids=lambda v: str(v))
-def test_ls_accumulate_fuzz(D, Ts):
+def test_ls_accumulate_fuzz(D, Ts, exact):
     st = LS(D)
     ref = ols.ls_state(D)
     for i, T in enumerate(Ts):
         a_loc, a_full = synth.make_activations(7000 + 31 * D + 7 * i + T, T, D)
         wsb = abi.ispa_ls_accumulate_workspace_size(D, T)
         ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
-        abi.ispa_ls_accumulate(st.c, bf16_tensor(a_loc), bf16_tensor(a_full), T, ws, wsb)
+        abi.ispa_ls_accumulate_ex(st.c, bf16_tensor(a_loc), bf16_tensor(a_full), T,
+                                  abi.ISPA_LS_EXACT_DELTA if exact else 0, ws, wsb)
         ols.ls_accumulate(ref, a_loc, a_full)
     torch.cuda.synchronize()
     assert st.c.n_tokens == sum(Ts)
