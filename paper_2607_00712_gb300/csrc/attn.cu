@@ -132,9 +132,6 @@ __device__ __forceinline__ void next_tile(const AttnParams& p, int& seg, int& of
   }
 }
 
-__device__ __forceinline__ void soft_barrier() {
-  asm volatile("bar.sync 1, %0;" ::"n"(N_SOFT) : "memory");
-}
 // Barriers of one softmax warp pair (the two warps of a TMEM lane quarter, 64 threads), ids
 // 2..5; pair_or also ORs a predicate over the pair.
 __device__ __forceinline__ void pair_sync(int id) {
@@ -601,17 +598,22 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
     auto warp_ok = [&](bool v) { return __all_sync(0xffffffffu, v); };
 
+    const int pair_id = 2 + quarter;   // named barrier of the warp pair (quarter, quarter + 4)
+    // The full row's l from the two column halves of the warp pair (block 0 of the exchange
+    // area, also used by the pair exchanges, which are complete on both sides of the pair
+    // before either warp gets here).  It does not depend on O, so the epilogue takes it before
+    // waiting for the last P V.  One pair barrier.
+    auto row_l = [&]() {
+      x_max[half * BM + row] = l_run;
+      pair_sync(pair_id);
+      return l_run + x_max[(half ^ 1) * BM + row];
+    };
     // Normalise O by the full-row l and store this warp's half of the row (bf16); optional
     // LSE; optional discrepancy partial sum_d (A_full - A_loc)^2 of this head on the stored
-    // bf16 values.  Executes the same two named barriers whether or not `live`.  Block 0 of
-    // the exchange area (also used by the pair exchanges, which are complete on both sides of
-    // the pair before either warp gets here) holds l, block 1 the squared sums.
-    auto emit = [&](bool live, __nv_bfloat16* dst, float* lse_dst, bool with_disc) {
-      float* x_l = x_max;             // [half][row]
+    // bf16 values.  Executes the same pair barrier whether or not `live`; after it both warps
+    // have read the l slots of row_l (block 0) and may reuse them.  Block 1 holds the squared sums.
+    auto emit = [&](bool live, float l_row, __nv_bfloat16* dst, float* lse_dst, bool with_disc) {
       float* x_sq = x_max + 2 * BM;   // [half][row]
-      x_l[half * BM + row] = l_run;
-      soft_barrier();
-      const float l_row = l_run + x_l[(half ^ 1) * BM + row];
       float sq = 0.f;
       if (live) {
         const float inv = (PV8 ? p.v_scale[head] : 1.f) / l_row;
@@ -649,7 +651,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // A warp that left through the abort path contributes NaN, so a row whose partial sum
       // is incomplete reaches disc (and the running sum of disc^2) as NaN, never as a value.
       x_sq[half * BM + row] = live ? sq : __int_as_float(0x7fc00000);
-      soft_barrier();
+      pair_sync(pair_id);
       if (row_ok && half == 0) {
         if (live && lse_dst)
           lse_dst[static_cast<size_t>(head) * p.n_q + qrow] =
@@ -659,7 +661,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
     };
 
-    const int pair_id = 2 + quarter;   // named barrier of the warp pair (quarter, quarter + 4)
     // O holds the item's tiles up to g once PV_g has completed: the commit that frees V_g's stage.
     auto wait_o = [&](int g, int site) {
       return warp_ok(mbar_wait(b.v_empty0 + 8 * (g % C::VST), (g / C::VST) & 1, wc, site, g));
@@ -764,9 +765,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int sb = g & 1;
         if (p.dual && j == p.n_local_tiles && j > 0) {
           // A_loc snapshot: O and l hold exactly the local tiles 0..j-1.
+          const float l_loc = row_l();
           if (ok) ok = wait_o(g - 1, 7);
           if (ok) tc_fence_after();
-          emit(ok, p.out_loc, p.lse_loc, false);
+          emit(ok, l_loc, p.out_loc, p.lse_loc, false);
         }
         if (ok) ok = warp_ok(mbar_wait(b.s_full0 + 8 * sb, (g >> 1) & 1, wc, 8, g));
         if (threadIdx.x == 0) tr(g, 0);
@@ -866,10 +868,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         next_tile(p, seg, off);
       }
       {
+        const float l_row = row_l();   // overlaps the last P V
         if (ok) ok = wait_o(base + n_tiles - 1, 11);
         if (ok) tc_fence_after();
-        if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, p.out_loc, p.lse_loc, false);
-        emit(ok, p.out, p.lse, p.dual != 0);
+        if (p.dual && p.n_local_tiles >= n_tiles) emit(ok, l_row, p.out_loc, p.lse_loc, false);
+        emit(ok, l_row, p.out, p.lse, p.dual != 0);
         if (threadIdx.x == 0 && k == 0) tr(0, 15);   // epilogue stored
       }
       // The next item's first PV (which overwrites O) waits for P'_0, which every softmax thread
