@@ -1056,7 +1056,22 @@ def cpu_baseline(wl, rows):
     return dict(value=round(flops / dt / 1e12, 6), unit=UNIT, cores=cores, kind="oracle",
                 sample=f"{rows} of {wl['nq']} query rows of each mode (full, local, dual) x all heads, "
                        f"plus LS accumulation of those rows; fp64 numpy, {dt:.1f} s",
-                seconds=round(dt, 2))
+                seconds=round(dt, 2), blas_threads=blas_threads())
+
+
+def blas_threads():
+    """Threads of numpy's BLAS as reported by threadpoolctl, else the environment's limit."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [d.get("num_threads") for d in threadpool_info() if d.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except Exception:   # threadpoolctl is optional
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return "library default (threadpoolctl not installed)"
 
 
 def run_reference(args, rank, world):
