@@ -76,8 +76,8 @@ def _check(st, ref, tol=1e-3):
 
 
 @pytest.mark.parametrize("exact", [False, True], ids=["scaled", "exact"])
-@pytest.mark.parametrize("D,Ts", [(128, [100]), (384, [64, 1999]), (512, [4680]), (1536, [4680, 37]),
-                                  (2048, [640])], ids=str)
+@pytest.mark.parametrize("D,Ts", [(128, [100]), (256, [1, 3]), (384, [64, 1999]), (512, [4680]),
+                                  (1536, [4680, 37]), (2048, [640])], ids=str)
 def test_both_forms_against_oracle(D, Ts, exact):
     st = LS(D)
     ref = ols.ls_state(D)
