@@ -716,27 +716,36 @@ __global__ void __launch_bounds__(W_THREADS, 1)
       const int row0 = (sg.kind == 2 ? D : 0) + sg.bi * 256 + half * 128 + quarter * 32;
       const int col0 = (sg.kind == 0 ? 0 : D) + sg.bj * 256;
       const float scale = p.unscale ? p.unscale[sg.kind] : 1.f;
+      // Two batches of four 32-column chunks: a batch's TMEM loads go out together, and the
+      // accumulator is handed back after the second batch's loads, waiting on the staging of
+      // three blocks instead of seven.
 #pragma unroll 1
-      for (int c = 0; c < 256 / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(lane_base + 32 * c, v);
-        tmem_wait_ld32(v);
-        if (c == 256 / 32 - 1) {
+      for (int hb = 0; hb < 2; ++hb) {
+        uint32_t v[4][32];
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) tmem_ld32(lane_base + 32 * (4 * hb + cc), v[cc]);
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) tmem_wait_ld32(v[cc]);
+        if (hb == 1) {
           tc_fence_before();
           mbar_arrive(acce0 + 8 * half);   // accumulator may be overwritten
         }
-        if (lane == 0) bulk_wait_read_all();   // the previous block's reduce has read the staging block
-        __syncwarp();
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-          tbuf[lane * 8 + (q ^ (lane & 7))] =
-              make_float4(__uint_as_float(v[4 * q]) * scale, __uint_as_float(v[4 * q + 1]) * scale,
-                          __uint_as_float(v[4 * q + 2]) * scale, __uint_as_float(v[4 * q + 3]) * scale);
-        fence_proxy_async_smem();   // these generic-proxy writes before the bulk copy reads them
-        __syncwarp();
-        if (lane == 0) {
-          tma_reduce_add_2d(&tm_state, tbuf_s, col0 + 32 * c, row0);
-          bulk_commit_group();
+        for (int cc = 0; cc < 4; ++cc) {
+          const int c = 4 * hb + cc;
+          if (lane == 0) bulk_wait_read_all();   // the previous block's reduce has read the staging block
+          __syncwarp();
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            tbuf[lane * 8 + (q ^ (lane & 7))] =
+                make_float4(__uint_as_float(v[cc][4 * q]) * scale, __uint_as_float(v[cc][4 * q + 1]) * scale,
+                            __uint_as_float(v[cc][4 * q + 2]) * scale, __uint_as_float(v[cc][4 * q + 3]) * scale);
+          fence_proxy_async_smem();   // these generic-proxy writes before the bulk copy reads them
+          __syncwarp();
+          if (lane == 0) {
+            tma_reduce_add_2d(&tm_state, tbuf_s, col0 + 32 * c, row0);
+            bulk_commit_group();
+          }
         }
       }
       ++m;
