@@ -655,8 +655,8 @@ ISPA_API ispa_status ispa_quantize_weight_e4m3(const float* W, const float* dW, 
 /* out: bf16 [T][D_out] = a_scale[t] * w_scale[n] * sum_k dec(a_q[t][k]) * dec(w_q[n][k]),
  * with a_q [T][D] and w_q [D_out][D] e4m3 codes from the two calls above, fp32
  * accumulation on the tensor cores, bf16 output (round to nearest).
- * D % 128 == 0 and D_out % 128 == 0 (else ISPA_ERR_UNSUPPORTED); a_q, w_q, out
- * 16-byte aligned. */
+ * D % 128 == 0 and D_out % 128 == 0 (else ISPA_ERR_UNSUPPORTED); a_q, w_q, w_scale
+ * and out 16-byte aligned. */
 ISPA_API ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uint8_t* w_q,
                                       const float* w_scale, int64_t T, int32_t D, int32_t D_out, void* out,
                                       ispa_stream stream);

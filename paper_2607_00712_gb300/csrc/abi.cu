@@ -784,7 +784,7 @@ ispa_status ispa_quantize_weight_e4m3(const float* W, const float* dW, int32_t D
 ispa_status ispa_linear_w8a8(const uint8_t* a_q, const float* a_scale, const uint8_t* w_q, const float* w_scale,
                              int64_t T, int32_t D, int32_t D_out, void* out, ispa_stream stream) {
   if (!a_q || !a_scale || !w_q || !w_scale || !out || T <= 0 || T > INT32_MAX || D <= 0 || D_out <= 0 ||
-      !aligned16(a_q) || !aligned16(w_q) || !aligned16(out))
+      !aligned16(a_q) || !aligned16(w_q) || !aligned16(w_scale) || !aligned16(out))
     return ISPA_ERR_INVALID_ARG;
   if (D % 128 != 0 || D_out % 128 != 0) return ISPA_ERR_UNSUPPORTED;
   int* status = device_status_ptr();

@@ -307,6 +307,17 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       __nv_bfloat16* orow = p.out + static_cast<size_t>(row) * p.Dout + n0;
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
+        // the 32 columns' weight scales (the same for every lane), loaded before the TMEM wait
+        float sw[32];
+        const float4* sw4 = reinterpret_cast<const float4*>(p.w_scale + n0 + 32 * c);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 t = sw4[q];
+          sw[4 * q] = t.x;
+          sw[4 * q + 1] = t.y;
+          sw[4 * q + 2] = t.z;
+          sw[4 * q + 3] = t.w;
+        }
         uint32_t v0[32], v1[32];
         tmem_ld32(taddr + 32 * c, v0);
         tmem_wait_ld32(v0);
@@ -315,7 +326,6 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           tmem_wait_ld32(v1);
         }
         if (row < p.T) {
-          const float* sw = p.w_scale + n0 + 32 * c;
           uint32_t pk[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {

@@ -175,6 +175,7 @@ def test_w8a8_validation_without_gpu():
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 100, 192, 256, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D % 128
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 100, 256, 192, 16, None) == abi.ISPA_ERR_UNSUPPORTED   # D_out % 128
     assert L.ispa_linear_w8a8(16, 16, 16, 16, 0, 256, 256, 16, None) == abi.ISPA_ERR_INVALID_ARG
+    assert L.ispa_linear_w8a8(16, 16, 16, 20, 10, 256, 256, 16, None) == abi.ISPA_ERR_INVALID_ARG   # w_scale
     assert L.ispa_linear_w8a8(24, 16, 16, 16, 10, 256, 256, 16, None) == abi.ISPA_ERR_INVALID_ARG    # misaligned
     assert L.ispa_quantize_rows_e4m3(16, 10, 24, 16, 16, None) == abi.ISPA_ERR_UNSUPPORTED           # cols % 16
     assert L.ispa_quantize_rows_e4m3(None, 10, 32, 16, 16, None) == abi.ISPA_ERR_INVALID_ARG
