@@ -224,15 +224,25 @@ __global__ void __launch_bounds__(256) amax_kernel(const uint4* __restrict__ a_l
   __shared__ float red[8];
   float ma = 0.f, md = 0.f;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
-    const uint4 a = a_loc[i], f = a_full[i];
-    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
+  // four words per thread and round, all loaded before any is used
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < n_words; i0 += 4 * stride) {
+    uint4 a[4], f[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
-      const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
-      ma = fmaxf(ma, fmaxf(fabsf(a0), fabsf(a1)));
-      md = fmaxf(md, fmaxf(fabsf(f0 - a0), fabsf(f1 - a1)));
+    for (int u = 0; u < 4; ++u) {
+      const int64_t i = i0 + u * stride;
+      a[u] = i < n_words ? a_loc[i] : make_uint4(0, 0, 0, 0);
+      f[u] = i < n_words ? a_full[i] : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t aw[4] = {a[u].x, a[u].y, a[u].z, a[u].w}, fw[4] = {f[u].x, f[u].y, f[u].z, f[u].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+        const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
+        ma = fmaxf(ma, fmaxf(fabsf(a0), fabsf(a1)));
+        md = fmaxf(md, fmaxf(fabsf(f0 - a0), fabsf(f1 - a1)));
+      }
     }
   }
   ma = block_max256(ma, red);
@@ -279,21 +289,35 @@ __global__ void __launch_bounds__(256) convert_kernel(const uint4* __restrict__ 
   pdl_trigger();   // the Gram kernel may set itself up meanwhile
   const float ka = pow2f(sa), kd = pow2f(sd);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride) {
-    const uint4 a = a_loc[i], f = a_full[i];
-    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, fw[4] = {f.x, f.y, f.z, f.w};
-    uint32_t ow[4], dw[4];
+  // four words per thread and round, all loaded before any is converted
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < n_words; i0 += 4 * stride) {
+    uint4 a[4], f[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
-      const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
-      __half2 h = __floats2half2_rn(a0 * ka, a1 * ka);
-      ow[e] = *reinterpret_cast<uint32_t*>(&h);
-      h = __floats2half2_rn((f0 - a0) * kd, (f1 - a1) * kd);
-      dw[e] = *reinterpret_cast<uint32_t*>(&h);
+    for (int u = 0; u < 4; ++u) {
+      const int64_t i = i0 + u * stride;
+      if (i < n_words) {
+        a[u] = a_loc[i];
+        f[u] = a_full[i];
+      }
     }
-    a16[i] = make_uint4(ow[0], ow[1], ow[2], ow[3]);
-    d16[i] = make_uint4(dw[0], dw[1], dw[2], dw[3]);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t i = i0 + u * stride;
+      if (i >= n_words) break;
+      const uint32_t aw[4] = {a[u].x, a[u].y, a[u].z, a[u].w}, fw[4] = {f[u].x, f[u].y, f[u].z, f[u].w};
+      uint32_t ow[4], dw[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+        const float f0 = __uint_as_float(fw[e] << 16), f1 = __uint_as_float(fw[e] & 0xFFFF0000u);
+        __half2 h = __floats2half2_rn(a0 * ka, a1 * ka);
+        ow[e] = *reinterpret_cast<uint32_t*>(&h);
+        h = __floats2half2_rn((f0 - a0) * kd, (f1 - a1) * kd);
+        dw[e] = *reinterpret_cast<uint32_t*>(&h);
+      }
+      a16[i] = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+      d16[i] = make_uint4(dw[0], dw[1], dw[2], dw[3]);
+    }
   }
 }
 
