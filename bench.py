@@ -59,7 +59,7 @@ def log(*a):
 # DRAM bytes of one F-layer attention launch of the 1.3B step (dram__bytes_read.sum +
 # dram__bytes_write.sum from one ncu capture of that launch), valid only for the kernel source
 # it was taken on: reported as null once attn.cu / ptx.cuh change.
-ATTN_TRAFFIC = {"source_sha256_16": "5844a3675d2795d7", "bytes": 239885824 + 11600384, "model": "1.3b"}
+ATTN_TRAFFIC = {"source_sha256_16": "a4d523e43ed3c924", "bytes": 242222592 + 11659008, "model": "1.3b"}
 
 
 def attn_source_sha():

@@ -12,6 +12,7 @@
 #include <stdint.h>
 
 #include "internal.h"
+#include "pdl.cuh"
 
 namespace ispa {
 
@@ -21,6 +22,7 @@ constexpr int kUnroll = 4;
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads) append_kernel(const AppendParams p) {
+  pdl_wait();   // the new K / V may come from the kernel before this one, which may still read the ring
   const int layer = blockIdx.y >> 1;
   const bool is_v = blockIdx.y & 1;
   const uint4* __restrict__ src =
@@ -68,8 +70,7 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   dim3 grid(static_cast<unsigned>(blocks), p.n_layers * 2);
-  append_kernel<<<grid, kThreads, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(append_kernel, grid, dim3(kThreads), 0, s, p);
 }
 
 }  // namespace ispa

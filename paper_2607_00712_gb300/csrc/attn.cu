@@ -930,36 +930,4 @@ cudaError_t launch_attention(int head_dim, const CUtensorMap* tq, const CUtensor
   return cudaErrorInvalidValue;
 }
 
-// ------------------------------------------------------------ discrepancy reduction
-// disc[t] = sqrt(sum_h part[h][t]);  *disc_sq_sum += sum over the block's tokens.
-__global__ void __launch_bounds__(256) disc_reduce_kernel(const float* __restrict__ part, int H,
-                                                          int n_q, float* __restrict__ disc,
-                                                          float* __restrict__ disc_sq_sum) {
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  float v = 0.f;
-  if (t < n_q) {
-    for (int h = 0; h < H; ++h) v += part[static_cast<size_t>(h) * n_q + t];
-    disc[t] = sqrtf(v);
-  }
-  __shared__ float red[8];
-  float w = v;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = w;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    w = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-    if (threadIdx.x == 0) atomicAdd(disc_sq_sum, w);
-  }
-}
-
-cudaError_t launch_disc_reduce(const float* part, int32_t H, int32_t n_q, float* disc,
-                               float* disc_sq_sum, cudaStream_t s) {
-  if (n_q <= 0) return cudaSuccess;
-  disc_reduce_kernel<<<(n_q + 255) / 256, 256, 0, s>>>(part, H, n_q, disc, disc_sq_sum);
-  return cudaGetLastError();
-}
-
 }  // namespace ispa

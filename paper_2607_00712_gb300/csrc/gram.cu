@@ -198,6 +198,7 @@ __global__ void __launch_bounds__(256) split_kernel(const uint4* __restrict__ a_
                                                     const uint4* __restrict__ a_full,
                                                     uint4* __restrict__ hi, uint4* __restrict__ lo,
                                                     int64_t n_words) {
+  pdl_wait();      // the inputs may come from the kernel before this one
   pdl_trigger();   // the Gram kernel after this one may set itself up meanwhile
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_words; i += stride)
@@ -220,6 +221,7 @@ __device__ __forceinline__ float block_max256(float v, float* red) {
 // Scaled form, pass 1: max |A_loc| and max |Delta| of each block's words -> part[b], part[nb + b].
 __global__ void __launch_bounds__(256) amax_kernel(const uint4* __restrict__ a_loc, const uint4* __restrict__ a_full,
                                                    int64_t n_words, float* __restrict__ part) {
+  pdl_wait();      // the inputs may come from the kernel before this one
   pdl_trigger();   // convert_kernel may set itself up meanwhile
   __shared__ float red[8];
   float ma = 0.f, md = 0.f;
@@ -920,19 +922,17 @@ cudaError_t launch_ls_accumulate(int32_t D, int64_t T, const void* a_loc, const 
   if (blocks > static_cast<int64_t>(sms) * 8) blocks = static_cast<int64_t>(sms) * 8;
   if (exact) {
     // hi, lo of Delta; the Gram kernel reads A_loc itself
-    split_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
-        static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), reinterpret_cast<uint4*>(op1),
-        reinterpret_cast<uint4*>(op2), n_words);
-    const cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_pdl(split_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s,
+                                     static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full),
+                                     reinterpret_cast<uint4*>(op1), reinterpret_cast<uint4*>(op2), n_words);
     if (e != cudaSuccess) return e;
     if (D % 256 == 0) return launch_gram_wide(D, T, 0, a_loc, op1, op2, nullptr, gram, status, wait_limit_ns, hb, s);
     return launch_gram<128>(D, T, 0, a_loc, op1, op2, nullptr, gram, status, wait_limit_ns, hb, s);
   }
   // scaled A_loc (op1) and Delta (op2) in fp16
   int nb = static_cast<int>(blocks < kAmaxBlocks ? blocks : kAmaxBlocks);
-  amax_kernel<<<static_cast<unsigned>(nb), 256, 0, s>>>(static_cast<const uint4*>(a_loc),
-                                                        static_cast<const uint4*>(a_full), n_words, part);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(amax_kernel, dim3(static_cast<unsigned>(nb)), dim3(256), 0, s,
+                             static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), n_words, part);
   if (e != cudaSuccess) return e;
   e = launch_pdl(convert_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s,
                  static_cast<const uint4*>(a_loc), static_cast<const uint4*>(a_full), n_words,

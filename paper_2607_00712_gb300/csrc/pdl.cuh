@@ -1,8 +1,8 @@
 // Programmatic dependent launch between kernels that follow each other on one stream: a
 // kernel launched with launch_pdl may start (and run its prologue: barrier set-up, TMEM
 // allocation) while the kernel before it finishes; it calls pdl_wait() before its first
-// access to global memory that the earlier kernel may write, which returns once that kernel
-// has completed and its writes are visible.  pdl_trigger() in the earlier kernel lets the
+// access to global memory that the earlier kernel may write (or, for a write of its own, may
+// still read), which returns once that kernel has completed and its writes are visible.  pdl_trigger() in the earlier kernel lets the
 // dependent start before all of its blocks have exited.
 #pragma once
 
