@@ -163,3 +163,24 @@ def test_back_to_back_accumulates_in_both_forms(D):
     torch.cuda.synchronize()
     assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
     _check(st, ref)
+
+
+def test_many_short_calls_alternating_forms():
+    # 40 calls of 1 to 130 tokens (ragged 64-token blocks, single-block and single-token calls),
+    # alternating the two forms, all on one stream before one synchronisation
+    D = 256
+    rng = np.random.default_rng(77)
+    st = LS(D)
+    ref = ols.ls_state(D)
+    keep = []
+    total = 0
+    for i in range(40):
+        T = int(rng.integers(1, 131))
+        a_loc, a_full = synth.make_activations(9300 + i, T, D)
+        ols.ls_accumulate(ref, a_loc, a_full)
+        keep.append(_accumulate(st, a_loc, a_full, exact=bool(i % 2)))
+        total += T
+    torch.cuda.synchronize()
+    assert abi.ispa_last_device_error()[0] == abi.ISPA_OK
+    assert st.c.n_tokens == total
+    _check(st, ref)
